@@ -1,0 +1,182 @@
+/*
+ * spire.h -- C ABI of libspire: the KV-cache-bound attention of one SPIRe
+ * speculation round (Neelam et al., "SPIRe: Boosting LLM Inference Throughput
+ * with Speculative Decoding", arXiv 2504.06419), on one NVIDIA GB300 (sm_103a).
+ *
+ * A speculation round is k draft-model passes followed by one target-model
+ * pass over the k+1 block tokens in parallel (Section 2, the Throughput
+ * Multiplier equation and the definitions of t_draft / t_verify beneath it;
+ * Fig. 1 caption).  In the large-batch long-context regime the cost of both is
+ * loading the KV cache (Section 1; Section 3.1).  This library implements that
+ * part:
+ *
+ *   spire_verify_attention        the target's verification attention: k+1
+ *                                 causal block queries per sequence over its
+ *                                 full, paged, ragged bf16 KV cache, with GQA.
+ *   spire_draft_sparse_attention  the draft's StreamingLLM attention: sink
+ *                                 entries plus a sliding window of feedback-
+ *                                 memory entries m_{<t} (Sections 3.1, 3.3),
+ *                                 over a bounded cache.
+ *
+ * Conventions common to every call
+ *   - All tensor arguments are DEVICE pointers, owned by the caller; the
+ *     library keeps no pointer after a call returns and allocates nothing.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
+ *     NULL is the legacy default stream).  Only spire_get_device_error
+ *     synchronises.
+ *   - Arguments that can be checked on the host are checked before anything is
+ *     launched; a failing check returns a status and launches nothing.
+ *   - Values that live on the device (ctx_lens, block_table) are checked by
+ *     the kernels.  A sequence whose values break the rules gets NaN in every
+ *     one of its output rows, and a bit is set in the device error word in the
+ *     workspace (read it with spire_get_device_error).  No kernel traps, reads
+ *     out of bounds or waits without a time limit.
+ *   - Results are deterministic: the split of the KV range across SMs depends
+ *     only on ctx_lens and the shapes, and the splits are merged in a fixed
+ *     order, so repeated calls give bit-identical outputs.
+ *   - Pointers to q, caches and out must be 16-byte aligned, the workspace
+ *     256-byte aligned.
+ */
+#ifndef SPIRE_H
+#define SPIRE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status of a host call. */
+typedef enum spire_status {
+    SPIRE_OK = 0,
+    SPIRE_ERR_INVALID_ARG = 1,  /* null pointer, bad shape, misalignment, ... */
+    SPIRE_ERR_UNSUPPORTED = 2,  /* valid but not implemented (head_dim, rows) */
+    SPIRE_ERR_WORKSPACE = 3,    /* workspace missing or smaller than required */
+    SPIRE_ERR_CUDA = 4          /* a CUDA runtime/driver call failed */
+} spire_status;
+
+/* Bits of the device error word (spire_get_device_error). */
+#define SPIRE_DEVERR_CTX_LEN 1u  /* a ctx_lens entry outside its allowed range */
+#define SPIRE_DEVERR_PAGE_ID 2u  /* a block_table entry outside [0, num_pages) */
+#define SPIRE_DEVERR_TIMEOUT 4u  /* a bounded wait inside a kernel gave up */
+
+/* Shapes shared by both kernels. */
+typedef struct spire_attn_desc {
+    int32_t batch;             /* B >= 0 sequences (B == 0: nothing to do) */
+    int32_t num_q_heads;       /* Hq >= 1 */
+    int32_t num_kv_heads;      /* Hkv >= 1, Hq % Hkv == 0; query head h reads
+                                  KV head h / (Hq / Hkv) (grouped-query) */
+    int32_t head_dim;          /* D, 64 or 128 */
+    int32_t page_size;         /* verify: tokens per KV page, must be 64 */
+    int32_t max_pages_per_seq; /* verify: columns of block_table */
+    int32_t num_pages;         /* verify: pages held by k_cache / v_cache */
+    float softmax_scale;       /* score = softmax_scale * <q, k>; finite, > 0
+                                  (1.0 when q is pre-scaled by 1/sqrt(D)) */
+} spire_attn_desc;
+
+/* Largest number of query rows one KV head serves: (Hq/Hkv) * (k+1) <= 128. */
+#define SPIRE_MAX_ROWS_PER_KV_HEAD 128
+
+/*
+ * spire_verify_workspace_bytes -- workspace size for spire_verify_attention.
+ * Depends only on the shapes (batch, heads, head_dim) and k, not on the
+ * device or on ctx_lens.  Returns 0 if desc is NULL or k < 0.
+ */
+size_t spire_verify_workspace_bytes(const spire_attn_desc *desc, int32_t k);
+
+/*
+ * spire_verify_attention -- verification attention of one speculation round
+ * (Section 2: t_verify is a target pass over the k+1 block tokens in
+ * parallel; Table 1 caption: a round yields 1..k+1 tokens).
+ *
+ *   q            bf16 [B, k+1, Hq, D]; block row i of sequence b.
+ *   k_cache      bf16 [num_pages, Hkv, page_size, D]; key of token j of
+ *                sequence b, KV head g, is
+ *                k_cache[block_table[b][j / page_size], g, j % page_size, :].
+ *   v_cache      bf16, same layout as k_cache.
+ *   block_table  int32 [B, max_pages_per_seq]; only the first
+ *                ceil(ctx_lens[b] / page_size) entries of row b are read, and
+ *                each must lie in [0, num_pages).
+ *   ctx_lens     int32 [B] on the device: L_b, the number of cache entries of
+ *                sequence b INCLUDING the k+1 block tokens, whose K/V the
+ *                caller has already written.  Must satisfy
+ *                k+1 <= L_b <= max_pages_per_seq * page_size.
+ *   k            speculation depth, k >= 0.
+ *   out          fp32 [B, k+1, Hq, D]:
+ *                out[b,i,h] = sum_j softmax_j(scale * <q[b,i,h], K_j>) V_j
+ *                over keys j < L_b - k + i (row i is causal within the block:
+ *                it equals single-query decoding at length L_b - k + i).
+ *   workspace    device buffer of >= spire_verify_workspace_bytes(desc, k)
+ *                bytes; holds the split plan, split partials and the device
+ *                error word.  Contents need no initialisation.  Calls that
+ *                share a workspace must be ordered (same stream).
+ * Returns SPIRE_OK once the work is enqueued.
+ */
+spire_status spire_verify_attention(const void *q, const void *k_cache,
+                                    const void *v_cache,
+                                    const int32_t *block_table,
+                                    const int32_t *ctx_lens, int32_t k,
+                                    const spire_attn_desc *desc, float *out,
+                                    void *workspace, size_t ws_bytes,
+                                    void *stream);
+
+/*
+ * spire_draft_workspace_bytes -- workspace size for
+ * spire_draft_sparse_attention.  Returns 0 for invalid arguments.
+ */
+size_t spire_draft_workspace_bytes(const spire_attn_desc *desc, int32_t n_sink,
+                                   int32_t window);
+
+/*
+ * spire_draft_sparse_attention -- one draft-model attention step with the
+ * StreamingLLM mask (Section 3.1: attention sink plus sliding window, a KV
+ * cache of constant size; Section 4: window 64, sink 1 in the paper) over
+ * feedback-memory entries (Section 3.3: z_t = Attention(x_t, m_{<t}); each
+ * draft layer keeps its own memory m^i, so each layer has its own cache).
+ *
+ *   q         bf16 [B, Hq, D]: one query per sequence.
+ *   kv        bf16 [B, 2, Hkv, S, D], S = n_sink + window; index 0 holds K,
+ *             1 holds V.  Memory entry p lives in slot spire_draft_slot(p):
+ *             sinks p < n_sink are fixed, later entries form a ring.
+ *   ctx_lens  int32 [B] on the device: t_b >= 1, the number of memory entries
+ *             m_0..m_{t-1} written so far.  The query sees
+ *             V(t) = {p < min(n_sink, t)} u {max(0, t - window) <= p < t},
+ *             which occupy exactly slots [0, min(t, S)).  The current token's
+ *             own entry is not visible (m_{<t}); pass t+1 after writing it for
+ *             self-inclusive StreamingLLM attention.
+ *   n_sink    >= 0 sink entries;  window >= 1 window entries.
+ *   out       fp32 [B, Hq, D].
+ *   workspace >= spire_draft_workspace_bytes(desc, n_sink, window) bytes.
+ * desc->page_size / max_pages_per_seq / num_pages are ignored.
+ */
+spire_status spire_draft_sparse_attention(const void *q, const void *kv,
+                                          const int32_t *ctx_lens,
+                                          int32_t n_sink, int32_t window,
+                                          const spire_attn_desc *desc,
+                                          float *out, void *workspace,
+                                          size_t ws_bytes, void *stream);
+
+/*
+ * spire_draft_slot -- slot of logical memory position p >= 0 in the bounded
+ * draft cache: p if p < n_sink, else n_sink + (p - n_sink) mod window.
+ * Returns -1 for p < 0, n_sink < 0 or window < 1.  Host function.
+ */
+int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
+
+/*
+ * spire_get_device_error -- copy the device error word of the most recent
+ * call that used `workspace` into *code_out (0 = no error, else an OR of
+ * SPIRE_DEVERR_* bits).  Synchronises `stream`.
+ */
+spire_status spire_get_device_error(const void *workspace, int32_t *code_out,
+                                    void *stream);
+
+/* spire_status_string -- static, human-readable name of a status. */
+const char *spire_status_string(spire_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPIRE_H */

@@ -1,0 +1,193 @@
+"""fp64 CPU oracle for SPIRe speculation-round attention (test infrastructure).
+
+This package is the slow, obviously correct reference the CUDA library is
+checked against.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import it.
+It shares no code with ``paper_2504_06419_gb300`` and never imports it.
+
+The arithmetic lives in ``spire_oracle.c`` (plain C, double precision, a
+pthread pool over independent (sequence, query head) units).  This module
+compiles it with gcc on first use and wraps it with ctypes.  Inputs are numpy
+arrays; bf16 tensors are passed as their raw 16-bit patterns (``uint16``).
+
+Functions (each follows the passage cited in ``spire_oracle.c``):
+  verify(...)          verification attention of the k+1 block tokens
+                       (Section 2: t_verify; Fig. 1 and Table 1 captions)
+  draft_ring(...)      sink + sliding-window attention over the bounded cache
+                       (Section 3.1, Section 3.3)
+  draft_logical(...)   the same mask over a full-length logical memory
+  ring_pack(...)       place logical memory entries into the bounded cache
+  draft_slot(p, ...)   slot of logical position p
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "spire_oracle.c")
+_LIB = os.path.join(_HERE, "libspire_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_F64 = ctypes.c_double
+
+
+def build(force: bool = False, src: str = _SRC, out: str = _LIB) -> str:
+    """Compile the oracle shared library with gcc (plain C11, -O2, pthreads)."""
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    tmp = out + ".tmp%d" % os.getpid()
+    cmd = ["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-pthread",
+           "-fno-fast-math", "-ffp-contract=off", "-o", tmp, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
+def _declare(lib):
+    lib.oracle_verify.restype = _I64
+    lib.oracle_verify.argtypes = [_P, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32,
+                                  _I32, _I32, _I32, _F64, _P, _P, _I32]
+    lib.oracle_draft_ring.restype = _I64
+    lib.oracle_draft_ring.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32,
+                                      _F64, _P, _P, _I32]
+    lib.oracle_draft_logical.restype = _I64
+    lib.oracle_draft_logical.argtypes = [_P, _P, _P, _P, _I32, _I32, _I32, _I32, _I64,
+                                         _I32, _I32, _F64, _P, _P, _I32]
+    lib.oracle_ring_pack.restype = _I64
+    lib.oracle_ring_pack.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I64, _I32, _I32, _P]
+    lib.oracle_draft_slot.restype = _I64
+    lib.oracle_draft_slot.argtypes = [_I64, _I32, _I32]
+    return lib
+
+
+def load(path: str | None = None):
+    """Load (building first if needed) the oracle library; returns a ctypes CDLL."""
+    global _lib
+    if path is not None:
+        return _declare(ctypes.CDLL(path))
+    with _lock:
+        if _lib is None:
+            _lib = _declare(ctypes.CDLL(build()))
+    return _lib
+
+
+def default_threads() -> int:
+    return max(1, os.cpu_count() or 1)
+
+
+def _u16(a) -> np.ndarray:
+    a = np.ascontiguousarray(a)
+    if a.dtype != np.uint16:
+        raise TypeError("bf16 inputs must be passed as uint16 bit patterns, got %s" % a.dtype)
+    return a
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def _ptr(a) -> int:
+    return a.ctypes.data if a is not None else None
+
+
+def _mask(unit_mask, n):
+    if unit_mask is None:
+        return None
+    m = np.ascontiguousarray(unit_mask, dtype=np.uint8).reshape(-1)
+    if m.size != n:
+        raise ValueError("unit_mask must have B*Hq entries")
+    return m
+
+
+def verify(q, k_cache, v_cache, block_table, ctx_lens, k, scale=1.0,
+           unit_mask=None, threads=None, lib=None):
+    """Verification attention, fp64.
+
+    q [B, k+1, Hq, D], k_cache / v_cache [num_pages, Hkv, page_size, D] (uint16
+    bf16 bits), block_table int32 [B, max_pages], ctx_lens int32 [B].
+    Returns (out float64 [B, k+1, Hq, D], n_bad_sequences).
+    """
+    lib = lib or load()
+    q, kc, vc = _u16(q), _u16(k_cache), _u16(v_cache)
+    bt, cl = _i32(block_table), _i32(ctx_lens)
+    B, rows, Hq, D = q.shape
+    if rows != k + 1:
+        raise ValueError("q must have k+1 rows")
+    num_pages, Hkv, page_size, D2 = kc.shape
+    if D2 != D or vc.shape != kc.shape:
+        raise ValueError("cache shape mismatch")
+    max_pages = bt.shape[1] if bt.ndim == 2 else 0
+    out = np.zeros((B, rows, Hq, D), dtype=np.float64)
+    m = _mask(unit_mask, B * Hq)
+    n_bad = lib.oracle_verify(_ptr(q), _ptr(kc), _ptr(vc), _ptr(bt), _ptr(cl), B, k, Hq,
+                              Hkv, D, page_size, max_pages, num_pages, float(scale),
+                              _ptr(m), _ptr(out), threads or default_threads())
+    if n_bad < 0:
+        raise ValueError("oracle_verify rejected its arguments")
+    return out, int(n_bad)
+
+
+def draft_ring(q, kv, ctx_lens, n_sink, window, scale=1.0, unit_mask=None,
+               threads=None, lib=None):
+    """Draft sink+window attention over the bounded cache kv [B, 2, Hkv, S, D]."""
+    lib = lib or load()
+    q, kv, cl = _u16(q), _u16(kv), _i32(ctx_lens)
+    B, Hq, D = q.shape
+    _, two, Hkv, S, D2 = kv.shape
+    if two != 2 or D2 != D or S != n_sink + window:
+        raise ValueError("kv must be [B, 2, Hkv, n_sink + window, D]")
+    out = np.zeros((B, Hq, D), dtype=np.float64)
+    m = _mask(unit_mask, B * Hq)
+    n_bad = lib.oracle_draft_ring(_ptr(q), _ptr(kv), _ptr(cl), B, Hq, Hkv, D, n_sink,
+                                  window, float(scale), _ptr(m), _ptr(out),
+                                  threads or default_threads())
+    if n_bad < 0:
+        raise ValueError("oracle_draft_ring rejected its arguments")
+    return out, int(n_bad)
+
+
+def draft_logical(q, k_log, v_log, ctx_lens, n_sink, window, scale=1.0,
+                  unit_mask=None, threads=None, lib=None):
+    """Draft attention over a full logical memory k_log / v_log [B, Hkv, T, D]."""
+    lib = lib or load()
+    q, kl, vl, cl = _u16(q), _u16(k_log), _u16(v_log), _i32(ctx_lens)
+    B, Hq, D = q.shape
+    _, Hkv, T, D2 = kl.shape
+    if D2 != D or vl.shape != kl.shape:
+        raise ValueError("logical cache shape mismatch")
+    out = np.zeros((B, Hq, D), dtype=np.float64)
+    m = _mask(unit_mask, B * Hq)
+    n_bad = lib.oracle_draft_logical(_ptr(q), _ptr(kl), _ptr(vl), _ptr(cl), B, Hq, Hkv, D,
+                                     T, n_sink, window, float(scale), _ptr(m), _ptr(out),
+                                     threads or default_threads())
+    if n_bad < 0:
+        raise ValueError("oracle_draft_logical rejected its arguments")
+    return out, int(n_bad)
+
+
+def ring_pack(k_log, v_log, ctx_lens, n_sink, window, kv_out=None, lib=None):
+    """Pack logical memory entries into a bounded cache; returns kv [B,2,Hkv,S,D]."""
+    lib = lib or load()
+    kl, vl, cl = _u16(k_log), _u16(v_log), _i32(ctx_lens)
+    B, Hkv, T, D = kl.shape
+    S = n_sink + window
+    if kv_out is None:
+        kv_out = np.zeros((B, 2, Hkv, S, D), dtype=np.uint16)
+    if lib.oracle_ring_pack(_ptr(kl), _ptr(vl), _ptr(cl), B, Hkv, D, T, n_sink, window,
+                            _ptr(kv_out)) != 0:
+        raise ValueError("oracle_ring_pack rejected its arguments")
+    return kv_out
+
+
+def draft_slot(p, n_sink, window, lib=None):
+    lib = lib or load()
+    return int(lib.oracle_draft_slot(int(p), int(n_sink), int(window)))

@@ -1,0 +1,411 @@
+/*
+ * spire_oracle.c -- plain fp64 CPU oracle for the attention of one SPIRe
+ * speculation round (Neelam et al., "SPIRe: Boosting LLM Inference Throughput
+ * with Speculative Decoding", arXiv 2504.06419).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously correct
+ * reference that the CUDA path is checked against.  Only the tests, the smoke
+ * check and the benchmark's CPU-baseline leg may load it.  It shares no code,
+ * header, table or helper with the CUDA library, and the CUDA library never
+ * calls it.
+ *
+ * Everything is computed in double precision.  bf16 inputs are widened
+ * exactly (a bf16 value is the top 16 bits of an IEEE binary32).  Softmax is
+ * two-pass: first the maximum score, then exp-sum and the weighted sum of
+ * values.  Keys are visited in increasing logical position.
+ *
+ * What each function follows:
+ *   oracle_verify      -- the verification pass of a speculation round:
+ *                         the target model runs on the k+1 block tokens in
+ *                         parallel (Section 2, definition of t_verify next to
+ *                         the Throughput Multiplier equation; Fig. 1 caption;
+ *                         Table 1 caption), each block token attending
+ *                         causally to the full KV cache (KV_target term of the
+ *                         implementation-agnostic multiplier, Section 2).
+ *   oracle_draft_*     -- the draft model's StreamingLLM attention mask:
+ *                         attention sinks plus a sliding window, so the draft
+ *                         KV cache has constant size (Section 3.1; Section 4,
+ *                         items 2 and 3), over feedback-memory entries m_{<t}
+ *                         (Section 3.3, the Feedback Transformer attention
+ *                         equation and the per-layer memory equation).
+ *   oracle_draft_slot  -- where logical memory position p lives in the
+ *                         bounded cache (sinks fixed, window a ring).
+ *
+ * Readings of points the paper leaves open (all listed in the design doc):
+ *   - scores are softmax_scale * <q, k>; the workloads pre-scale q, scale = 1;
+ *   - verify ctx_lens[b] = L counts the cache entries including the k+1 block
+ *     tokens; block row i (0..k) sees keys j < L - k + i;
+ *   - GQA: query head h uses KV head h / (Hq / Hkv);
+ *   - draft ctx_lens[b] = t is the number of memory entries m_0..m_{t-1};
+ *     the visible set is V(t) = {p < min(n_sink, t)} u {max(0, t-window) <= p < t};
+ *   - a sequence whose length breaks the rules (verify: L < k+1 or
+ *     L > max_pages*page_size; draft: t < 1) or whose block table points
+ *     outside the cache gets NaN in all of its output rows and the function
+ *     returns a nonzero count of such sequences.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ---- exact bf16 -> double ---------------------------------------------- */
+static double bf16_to_double(uint16_t bits)
+{
+    uint32_t u = (uint32_t)bits << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* ---- one softmax-weighted average over an explicit key list -------------
+ * keys[j] / vals[j] point at D bf16 values; n >= 1.  out[d] receives
+ * sum_j p_j v_j[d] with p = softmax(scale * <q, k_j>), two passes. */
+static void attend(const uint16_t *q, const uint16_t *const *keys,
+                   const uint16_t *const *vals, int64_t n, int32_t D,
+                   double scale, double *scores, double *out)
+{
+    double m = -INFINITY;
+    for (int64_t j = 0; j < n; ++j) {
+        double s = 0.0;
+        for (int32_t d = 0; d < D; ++d)
+            s += bf16_to_double(q[d]) * bf16_to_double(keys[j][d]);
+        s *= scale;
+        scores[j] = s;
+        if (s > m)
+            m = s;
+    }
+    double l = 0.0;
+    for (int32_t d = 0; d < D; ++d)
+        out[d] = 0.0;
+    for (int64_t j = 0; j < n; ++j) {
+        double p = exp(scores[j] - m);
+        l += p;
+        for (int32_t d = 0; d < D; ++d)
+            out[d] += p * bf16_to_double(vals[j][d]);
+    }
+    for (int32_t d = 0; d < D; ++d)
+        out[d] /= l;
+}
+
+/* ---- a tiny thread pool over independent (b, h) units ------------------- */
+typedef void (*unit_fn)(void *ctx, int64_t unit, double *scores,
+                        const uint16_t **keys, const uint16_t **vals);
+
+typedef struct {
+    unit_fn fn;
+    void *ctx;
+    int64_t n_units;
+    int64_t max_keys;
+    const uint8_t *unit_mask;
+    int64_t next;
+    pthread_mutex_t lock;
+} pool_t;
+
+static void *pool_worker(void *arg)
+{
+    pool_t *p = (pool_t *)arg;
+    int64_t cap = p->max_keys > 0 ? p->max_keys : 1;
+    double *scores = (double *)malloc(sizeof(double) * (size_t)cap);
+    const uint16_t **keys = (const uint16_t **)malloc(sizeof(void *) * (size_t)cap);
+    const uint16_t **vals = (const uint16_t **)malloc(sizeof(void *) * (size_t)cap);
+    if (!scores || !keys || !vals) {
+        free(scores); free((void *)keys); free((void *)vals);
+        return (void *)1;
+    }
+    for (;;) {
+        pthread_mutex_lock(&p->lock);
+        int64_t u = p->next++;
+        pthread_mutex_unlock(&p->lock);
+        if (u >= p->n_units)
+            break;
+        if (p->unit_mask && !p->unit_mask[u])
+            continue;
+        p->fn(p->ctx, u, scores, keys, vals);
+    }
+    free(scores); free((void *)keys); free((void *)vals);
+    return NULL;
+}
+
+static int run_pool(unit_fn fn, void *ctx, int64_t n_units, int64_t max_keys,
+                    const uint8_t *unit_mask, int32_t n_threads)
+{
+    pool_t p = {fn, ctx, n_units, max_keys, unit_mask, 0, PTHREAD_MUTEX_INITIALIZER};
+    if (n_threads < 1)
+        n_threads = 1;
+    if (n_threads > 1024)
+        n_threads = 1024;
+    pthread_t tids[1024];
+    int started = 0, failed = 0;
+    for (int i = 0; i < n_threads; ++i) {
+        if (pthread_create(&tids[i], NULL, pool_worker, &p) != 0)
+            break;
+        ++started;
+    }
+    if (started == 0) {
+        if (pool_worker(&p) != NULL)
+            failed = 1;
+    }
+    for (int i = 0; i < started; ++i) {
+        void *ret = NULL;
+        pthread_join(tids[i], &ret);
+        if (ret != NULL)
+            failed = 1;
+    }
+    return failed ? -1 : 0;
+}
+
+/* ======================================================================== */
+/* Verification attention                                                    */
+/* ======================================================================== */
+typedef struct {
+    const uint16_t *q, *k_cache, *v_cache;
+    const int32_t *block_table, *ctx_lens;
+    int32_t B, k, Hq, Hkv, D, page_size, max_pages, num_pages;
+    double scale;
+    double *out;
+    int32_t *bad;           /* per sequence: 1 if its lengths/pages break the rules */
+} verify_ctx;
+
+/* Index of key j of sequence b, KV head g, inside a [num_pages, Hkv, P, D]
+ * cache, through the block table.  Returns NULL for a page id outside the
+ * cache. */
+static const uint16_t *paged_row(const verify_ctx *c, const uint16_t *cache,
+                                 int32_t b, int32_t g, int64_t j)
+{
+    int64_t page = c->block_table[(int64_t)b * c->max_pages + j / c->page_size];
+    if (page < 0 || page >= c->num_pages)
+        return NULL;
+    int64_t slot = j % c->page_size;
+    return cache + (((page * c->Hkv + g) * c->page_size + slot) * c->D);
+}
+
+static void verify_unit(void *vctx, int64_t unit, double *scores,
+                        const uint16_t **keys, const uint16_t **vals)
+{
+    verify_ctx *c = (verify_ctx *)vctx;
+    int32_t b = (int32_t)(unit / c->Hq);
+    int32_t h = (int32_t)(unit % c->Hq);
+    int32_t group = c->Hq / c->Hkv;
+    int32_t g = h / group;
+    int64_t L = c->ctx_lens[b];
+    int32_t rows = c->k + 1;
+    int valid = L >= rows && L <= (int64_t)c->max_pages * c->page_size;
+    for (int32_t i = 0; valid && i < rows; ++i) {
+        int64_t n_i = L - c->k + i;            /* keys visible to block row i */
+        for (int64_t j = 0; j < n_i; ++j) {
+            keys[j] = paged_row(c, c->k_cache, b, g, j);
+            vals[j] = paged_row(c, c->v_cache, b, g, j);
+            if (!keys[j] || !vals[j]) {
+                valid = 0;
+                break;
+            }
+        }
+        if (!valid)
+            break;
+        const uint16_t *qi = c->q + (((int64_t)b * rows + i) * c->Hq + h) * c->D;
+        double *oi = c->out + (((int64_t)b * rows + i) * c->Hq + h) * c->D;
+        attend(qi, keys, vals, n_i, c->D, c->scale, scores, oi);
+    }
+    if (!valid) {
+        c->bad[b] = 1;
+        for (int32_t i = 0; i < rows; ++i) {
+            double *oi = c->out + (((int64_t)b * rows + i) * c->Hq + h) * c->D;
+            for (int32_t d = 0; d < c->D; ++d)
+                oi[d] = NAN;
+        }
+    }
+}
+
+/*
+ * oracle_verify: out[b, i, h, :] for b < B, block row i <= k, query head h.
+ *   q        bf16 bits [B, k+1, Hq, D]
+ *   k_cache  bf16 bits [num_pages, Hkv, page_size, D]   (v_cache alike)
+ *   block_table int32 [B, max_pages]; ctx_lens int32 [B]
+ *   unit_mask  NULL, or uint8 [B*Hq]: compute only (b, h) with mask != 0
+ *              (other outputs are left untouched)
+ *   out        double [B, k+1, Hq, D]
+ * Returns the number of sequences whose inputs break the rules (their rows
+ * are NaN), or -1 on bad arguments / allocation failure.
+ */
+int64_t oracle_verify(const uint16_t *q, const uint16_t *k_cache,
+                      const uint16_t *v_cache, const int32_t *block_table,
+                      const int32_t *ctx_lens, int32_t B, int32_t k, int32_t Hq,
+                      int32_t Hkv, int32_t D, int32_t page_size,
+                      int32_t max_pages, int32_t num_pages, double scale,
+                      const uint8_t *unit_mask, double *out, int32_t n_threads)
+{
+    if (B < 0 || k < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || D < 1 ||
+        page_size < 1 || max_pages < 0 || num_pages < 0)
+        return -1;
+    if (B == 0)
+        return 0;
+    int32_t *bad = (int32_t *)calloc((size_t)B, sizeof(int32_t));
+    if (!bad)
+        return -1;
+    verify_ctx c = {q, k_cache, v_cache, block_table, ctx_lens, B, k, Hq, Hkv,
+                    D, page_size, max_pages, num_pages, scale, out, bad};
+    int64_t max_keys = (int64_t)max_pages * page_size;
+    int rc = run_pool(verify_unit, &c, (int64_t)B * Hq, max_keys, unit_mask, n_threads);
+    int64_t n_bad = 0;
+    for (int32_t b = 0; b < B; ++b)
+        n_bad += bad[b];
+    free(bad);
+    return rc ? -1 : n_bad;
+}
+
+/* ======================================================================== */
+/* Draft static sparse attention                                             */
+/* ======================================================================== */
+
+/* Slot of logical memory position p in a cache of n_sink fixed slots followed
+ * by a ring of `window` slots. */
+int64_t oracle_draft_slot(int64_t p, int32_t n_sink, int32_t window)
+{
+    if (p < n_sink)
+        return p;
+    return n_sink + (p - n_sink) % window;
+}
+
+/* Membership of logical position p in V(t): the first n_sink entries and the
+ * last `window` entries of m_0..m_{t-1}. */
+static int visible(int64_t p, int64_t t, int32_t n_sink, int32_t window)
+{
+    if (p < 0 || p >= t)
+        return 0;
+    return p < n_sink || p >= t - window;
+}
+
+typedef struct {
+    const uint16_t *q;
+    const uint16_t *k_src, *v_src;   /* logical [B,Hkv,T,D] x2, or ring [B,2,Hkv,S,D] */
+    int ring;
+    const int32_t *ctx_lens;
+    int32_t B, Hq, Hkv, D, n_sink, window;
+    int64_t T;                        /* logical length capacity (logical form) */
+    double scale;
+    double *out;
+    int32_t *bad;
+} draft_ctx;
+
+static void draft_unit(void *vctx, int64_t unit, double *scores,
+                       const uint16_t **keys, const uint16_t **vals)
+{
+    draft_ctx *c = (draft_ctx *)vctx;
+    int32_t b = (int32_t)(unit / c->Hq);
+    int32_t h = (int32_t)(unit % c->Hq);
+    int32_t g = h / (c->Hq / c->Hkv);
+    int64_t t = c->ctx_lens[b];
+    int64_t S = (int64_t)c->n_sink + c->window;
+    double *o = c->out + ((int64_t)b * c->Hq + h) * c->D;
+    int ok = t >= 1 && (c->ring || t <= c->T);
+    int64_t n = 0;
+    for (int64_t p = 0; ok && p < t; ++p) {
+        if (!visible(p, t, c->n_sink, c->window))
+            continue;
+        if (c->ring) {
+            int64_t s = oracle_draft_slot(p, c->n_sink, c->window);
+            const uint16_t *base = c->k_src;  /* ring: k_src holds the whole [B,2,Hkv,S,D] */
+            keys[n] = base + ((((int64_t)b * 2 + 0) * c->Hkv + g) * S + s) * c->D;
+            vals[n] = base + ((((int64_t)b * 2 + 1) * c->Hkv + g) * S + s) * c->D;
+        } else {
+            keys[n] = c->k_src + (((int64_t)b * c->Hkv + g) * c->T + p) * c->D;
+            vals[n] = c->v_src + (((int64_t)b * c->Hkv + g) * c->T + p) * c->D;
+        }
+        ++n;
+    }
+    if (!ok || n == 0) {
+        c->bad[b] = 1;
+        for (int32_t d = 0; d < c->D; ++d)
+            o[d] = NAN;
+        return;
+    }
+    attend(c->q + ((int64_t)b * c->Hq + h) * c->D, keys, vals, n, c->D,
+           c->scale, scores, o);
+}
+
+static int64_t draft_common(draft_ctx *c, const uint8_t *unit_mask,
+                            int32_t n_threads, int64_t max_keys)
+{
+    if (c->B < 0 || c->Hq < 1 || c->Hkv < 1 || c->Hq % c->Hkv != 0 ||
+        c->D < 1 || c->n_sink < 0 || c->window < 1)
+        return -1;
+    if (c->B == 0)
+        return 0;
+    c->bad = (int32_t *)calloc((size_t)c->B, sizeof(int32_t));
+    if (!c->bad)
+        return -1;
+    int rc = run_pool(draft_unit, c, (int64_t)c->B * c->Hq, max_keys, unit_mask, n_threads);
+    int64_t n_bad = 0;
+    for (int32_t b = 0; b < c->B; ++b)
+        n_bad += c->bad[b];
+    free(c->bad);
+    return rc ? -1 : n_bad;
+}
+
+/*
+ * oracle_draft_logical: the definition over a full-length logical memory.
+ *   q       bf16 bits [B, Hq, D] (one draft query per sequence)
+ *   k_log   bf16 bits [B, Hkv, T, D]: K of memory entries m_0..m_{T-1}
+ *   v_log   bf16 bits [B, Hkv, T, D]
+ *   ctx_lens int32 [B]: t, the number of memory entries the query may see
+ *   out     double [B, Hq, D]
+ */
+int64_t oracle_draft_logical(const uint16_t *q, const uint16_t *k_log,
+                             const uint16_t *v_log, const int32_t *ctx_lens,
+                             int32_t B, int32_t Hq, int32_t Hkv, int32_t D,
+                             int64_t T, int32_t n_sink, int32_t window,
+                             double scale, const uint8_t *unit_mask,
+                             double *out, int32_t n_threads)
+{
+    draft_ctx c = {q, k_log, v_log, 0, ctx_lens, B, Hq, Hkv, D, n_sink, window,
+                   T, scale, out, NULL};
+    return draft_common(&c, unit_mask, n_threads, T);
+}
+
+/*
+ * oracle_draft_ring: the same visible set V(t), each entry read from its slot
+ * of the bounded cache.
+ *   kv   bf16 bits [B, 2, Hkv, n_sink + window, D]  (index 0 = K, 1 = V)
+ */
+int64_t oracle_draft_ring(const uint16_t *q, const uint16_t *kv,
+                          const int32_t *ctx_lens, int32_t B, int32_t Hq,
+                          int32_t Hkv, int32_t D, int32_t n_sink,
+                          int32_t window, double scale,
+                          const uint8_t *unit_mask, double *out,
+                          int32_t n_threads)
+{
+    draft_ctx c = {q, kv, NULL, 1, ctx_lens, B, Hq, Hkv, D, n_sink, window,
+                   0, scale, out, NULL};
+    return draft_common(&c, unit_mask, n_threads, (int64_t)n_sink + window);
+}
+
+/*
+ * oracle_ring_pack: write memory entries m_0..m_{t_b - 1} of a logical cache
+ * into the bounded cache in order of increasing position, each to its slot
+ * (a later entry overwrites an earlier one in the same ring slot).  Slots
+ * never written are left untouched.
+ */
+int64_t oracle_ring_pack(const uint16_t *k_log, const uint16_t *v_log,
+                         const int32_t *ctx_lens, int32_t B, int32_t Hkv,
+                         int32_t D, int64_t T, int32_t n_sink, int32_t window,
+                         uint16_t *kv)
+{
+    if (B < 0 || Hkv < 1 || D < 1 || n_sink < 0 || window < 1)
+        return -1;
+    int64_t S = (int64_t)n_sink + window;
+    for (int32_t b = 0; b < B; ++b) {
+        int64_t t = ctx_lens[b];
+        if (t > T)
+            return -1;
+        for (int32_t g = 0; g < Hkv; ++g)
+            for (int64_t p = 0; p < t; ++p) {
+                int64_t s = oracle_draft_slot(p, n_sink, window);
+                const uint16_t *ks = k_log + (((int64_t)b * Hkv + g) * T + p) * D;
+                const uint16_t *vs = v_log + (((int64_t)b * Hkv + g) * T + p) * D;
+                memcpy(kv + ((((int64_t)b * 2 + 0) * Hkv + g) * S + s) * D, ks, sizeof(uint16_t) * D);
+                memcpy(kv + ((((int64_t)b * 2 + 1) * Hkv + g) * S + s) * D, vs, sizeof(uint16_t) * D);
+            }
+    }
+    return 0;
+}

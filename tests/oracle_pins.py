@@ -1,0 +1,371 @@
+"""Pins of the fp64 oracle against facts the paper's definitions and plain
+mathematics fix -- not against the oracle itself.
+
+Every pin takes the ctypes handle of an oracle build, so the same pins run on
+the real oracle (test_oracle_pins.py) and on deliberately broken copies of it
+(test_oracle_mutants.py), which shows each plausible mistake trips a pin.
+
+What fixes each expected value:
+  * closed forms: with q = 0 every visible key has the same weight, so the
+    output is the exact arithmetic mean of the visible values; if value j
+    encodes its own logical position, that mean is a closed-form function of
+    the visible set (verify: positions 0..L-k+i-1; draft: sinks plus window);
+  * a two-key softmax is the logistic function;
+  * a library routine: torch's fp64 scaled_dot_product_attention with an
+    explicit boolean mask;
+  * invariants the definitions imply: constant V, one dominant logit,
+    row i == decoding at length L-k+i, window >= t == full attention,
+    causality, page-permutation invariance, ring packing == logical mask.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import oracle
+import workloads
+
+PAGE = 64
+
+
+def _f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Exact for values representable in bf16 (small integers, powers of 2)."""
+    t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16)
+    rt = t.to(torch.float32).numpy()
+    assert np.array_equal(rt, np.asarray(x, dtype=np.float32)), "value not exact in bf16"
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def _bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _paged_from_logical(Kl, Vl, L, rng, page=PAGE):
+    """Scatter logical per-sequence K/V [B, Hkv, T, D] (bits) into a shuffled
+    paged cache; returns (k_cache, v_cache, block_table)."""
+    B, Hkv, T, D = Kl.shape
+    pages = [(int(l) + page - 1) // page for l in L]
+    n = sum(pages)
+    order = rng.permutation(n)
+    bt = np.full((B, max(pages)), -1, dtype=np.int32)
+    kc = np.zeros((n, Hkv, page, D), dtype=np.uint16)
+    vc = np.zeros_like(kc)
+    off = 0
+    for b in range(B):
+        for p in range(pages[b]):
+            phys = order[off + p]
+            bt[b, p] = phys
+            lo, hi = p * page, min((p + 1) * page, int(L[b]))
+            kc[phys, :, :hi - lo] = Kl[b, :, lo:hi]
+            vc[phys, :, :hi - lo] = Vl[b, :, lo:hi]
+        off += pages[b]
+    return kc, vc, bt
+
+
+# --------------------------------------------------------------------------
+# verify pins
+# --------------------------------------------------------------------------
+def pin_verify_uniform_logits_closed_form(lib):
+    """q = 0: row i of sequence b, head h returns the mean of the values at
+    logical positions 0..L-k+i-1.  Value j carries (j, kv-head index, 1, 0)."""
+    rng = np.random.default_rng(11)
+    k, Hq, Hkv, D = 3, 6, 3, 4
+    G = Hq // Hkv
+    L = np.array([4, 64, 65, 130, 200], dtype=np.int32)
+    B, T = len(L), int(L.max())
+    Kl = _f32_to_bf16_bits(rng.integers(-3, 4, size=(B, Hkv, T, D)).astype(np.float32))
+    vals = np.zeros((B, Hkv, T, D), dtype=np.float32)
+    vals[..., 0] = np.arange(T)[None, None, :]
+    vals[..., 1] = np.arange(Hkv)[None, :, None]
+    vals[..., 2] = 1.0
+    Vl = _f32_to_bf16_bits(vals)
+    kc, vc, bt = _paged_from_logical(Kl, Vl, L, rng)
+    q = np.zeros((B, k + 1, Hq, D), dtype=np.uint16)
+    out, n_bad = oracle.verify(q, kc, vc, bt, L, k, lib=lib)
+    assert n_bad == 0
+    for b in range(B):
+        for i in range(k + 1):
+            n = int(L[b]) - k + i
+            for h in range(Hq):
+                exp = np.array([(n - 1) / 2.0, h // G, 1.0, 0.0])
+                np.testing.assert_allclose(out[b, i, h], exp, rtol=0, atol=1e-12)
+
+
+def pin_verify_two_key_logistic(lib):
+    """Two visible keys with scores a*scale and 0: weights are the logistic
+    function of a*scale."""
+    D = 2
+    for a, scale in [(1.0, 1.0), (2.0, 0.5), (-3.0, 1.0)]:
+        q = _f32_to_bf16_bits(np.array([[[[a, 0.0]]]], dtype=np.float32))
+        keys = np.array([[1.0, 0.0], [0.0, 1.0]], dtype=np.float32)
+        vals = np.array([[2.0, -1.0], [0.5, 4.0]], dtype=np.float32)
+        kc = np.zeros((1, 1, PAGE, D), dtype=np.uint16)
+        vc = np.zeros_like(kc)
+        kc[0, 0, :2] = _f32_to_bf16_bits(keys)
+        vc[0, 0, :2] = _f32_to_bf16_bits(vals)
+        bt = np.zeros((1, 1), dtype=np.int32)
+        out, _ = oracle.verify(q, kc, vc, bt, np.array([2], np.int32), 0, scale=scale, lib=lib)
+        w0 = 1.0 / (1.0 + math.exp(-a * scale))
+        exp = w0 * vals[0].astype(np.float64) + (1.0 - w0) * vals[1].astype(np.float64)
+        np.testing.assert_allclose(out[0, 0, 0], exp, rtol=1e-14, atol=1e-14)
+
+
+def pin_verify_constant_v(lib):
+    """V identically c returns c for every row."""
+    rng = np.random.default_rng(12)
+    vi = workloads.make_verify([9, 70, 129], 2, 4, 2, 8, seed=5, device="cpu")
+    c = 0.8125
+    vc = workloads.bf16_bits(torch.full_like(vi.v_cache, c))
+    out, _ = oracle.verify(workloads.bf16_bits(vi.q), workloads.bf16_bits(vi.k_cache), vc,
+                           vi.block_table.numpy(), vi.ctx_lens.numpy(), vi.k, lib=lib)
+    np.testing.assert_allclose(out, c, rtol=0, atol=1e-15)
+    del rng
+
+
+def pin_verify_one_hot_logit(lib):
+    """One key whose score exceeds all others by >= 60 yields its value (the
+    others carry weight < e^-60)."""
+    D, L = 4, 50
+    q = _f32_to_bf16_bits(np.array([[[[16.0, 0, 0, 0]]]], dtype=np.float32))
+    keys = np.zeros((L, D), np.float32)
+    keys[:, 1] = 1.0
+    keys[17, 0] = 4.0        # score 64 vs 0
+    rng = np.random.default_rng(13)
+    vals = rng.integers(-8, 9, size=(L, D)).astype(np.float32)
+    kc = np.zeros((1, 1, PAGE, D), np.uint16)
+    vc = np.zeros_like(kc)
+    kc[0, 0, :L] = _f32_to_bf16_bits(keys)
+    vc[0, 0, :L] = _f32_to_bf16_bits(vals)
+    out, _ = oracle.verify(q, kc, vc, np.zeros((1, 1), np.int32), np.array([L], np.int32), 0,
+                           lib=lib)
+    np.testing.assert_allclose(out[0, 0, 0], vals[17], rtol=0, atol=1e-20 + 64 * math.exp(-60))
+
+
+def pin_verify_matches_sdpa(lib):
+    """torch fp64 scaled_dot_product_attention with an explicit causal-block
+    mask and GQA head expansion, on random data."""
+    for (L, k, Hq, Hkv, D, scale, seed) in [([7, 64, 100], 2, 4, 2, 16, 1.0, 1),
+                                              ([5, 128], 4, 3, 1, 8, 0.37, 2),
+                                              ([1, 66], 0, 2, 2, 32, 1.0, 3)]:
+        vi = workloads.make_verify(L, k, Hq, Hkv, D, seed=seed, device="cpu", shuffle=True)
+        qb, kb, vb = (workloads.bf16_bits(t) for t in (vi.q, vi.k_cache, vi.v_cache))
+        out, n_bad = oracle.verify(qb, kb, vb, vi.block_table.numpy(), vi.ctx_lens.numpy(), k,
+                                   scale=scale, lib=lib)
+        assert n_bad == 0
+        G = Hq // Hkv
+        for b, Lb in enumerate(L):
+            pages = vi.block_table[b, :(Lb + PAGE - 1) // PAGE].long()
+            K = vi.k_cache[pages].permute(1, 0, 2, 3).reshape(Hkv, -1, D)[:, :Lb].double()
+            V = vi.v_cache[pages].permute(1, 0, 2, 3).reshape(Hkv, -1, D)[:, :Lb].double()
+            K = K.repeat_interleave(G, dim=0)
+            V = V.repeat_interleave(G, dim=0)
+            Q = vi.q[b].permute(1, 0, 2).double()               # [Hq, k+1, D]
+            rows = torch.arange(k + 1)[:, None]
+            cols = torch.arange(Lb)[None, :]
+            mask = cols < (Lb - k + rows)
+            ref = torch.nn.functional.scaled_dot_product_attention(
+                Q, K, V, attn_mask=mask, scale=scale)            # [Hq, k+1, D]
+            np.testing.assert_allclose(out[b], ref.permute(1, 0, 2).numpy(), rtol=1e-12,
+                                       atol=1e-12)
+
+
+def pin_verify_row_equals_decode(lib):
+    """Block row i equals single-query decoding (k = 0) at length L-k+i."""
+    L, k = [70, 131], 4
+    vi = workloads.make_verify(L, k, 4, 2, 16, seed=21, device="cpu")
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (vi.q, vi.k_cache, vi.v_cache))
+    bt = vi.block_table.numpy()
+    out, _ = oracle.verify(qb, kb, vb, bt, np.array(L, np.int32), k, lib=lib)
+    for i in range(k + 1):
+        Li = np.array([l - k + i for l in L], np.int32)
+        dec, _ = oracle.verify(np.ascontiguousarray(qb[:, i:i + 1]), kb, vb, bt, Li, 0, lib=lib)
+        np.testing.assert_allclose(out[:, i], dec[:, 0], rtol=1e-15, atol=1e-15)
+
+
+def pin_verify_causality(lib):
+    """Changing the K/V of block token at position L-k+i changes row i and
+    leaves rows < i bit-identical."""
+    L, k = [100], 4
+    vi = workloads.make_verify(L, k, 2, 1, 8, seed=31, device="cpu", shuffle=False)
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (vi.q, vi.k_cache, vi.v_cache))
+    bt = vi.block_table.numpy()
+    base, _ = oracle.verify(qb, kb, vb, bt, np.array(L, np.int32), k, lib=lib)
+    for i in range(1, k + 1):
+        j = L[0] - k + i - 1          # first key visible to row i but not row i-1
+        kb2, vb2 = kb.copy(), vb.copy()
+        page, slot = bt[0, j // PAGE], j % PAGE
+        kb2[page, :, slot] = _f32_to_bf16_bits(np.full(8, 2.0, np.float32))
+        vb2[page, :, slot] = _f32_to_bf16_bits(np.full(8, 64.0, np.float32))
+        out, _ = oracle.verify(qb, kb2, vb2, bt, np.array(L, np.int32), k, lib=lib)
+        assert np.array_equal(out[:, :i], base[:, :i])
+        assert not np.allclose(out[:, i], base[:, i])
+
+
+def pin_verify_page_permutation(lib):
+    """Permuting physical pages (and the block table with them) gives
+    bit-identical results."""
+    L, k = [130, 64, 3], 1
+    vi = workloads.make_verify(L, k, 4, 2, 8, seed=41, device="cpu", shuffle=False)
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (vi.q, vi.k_cache, vi.v_cache))
+    bt = vi.block_table.numpy()
+    base, _ = oracle.verify(qb, kb, vb, bt, np.array(L, np.int32), k, lib=lib)
+    perm = np.random.default_rng(3).permutation(kb.shape[0])
+    inv = np.argsort(perm)
+    bt2 = np.where(bt >= 0, inv[np.maximum(bt, 0)], -1).astype(np.int32)
+    out, _ = oracle.verify(qb, kb[perm], vb[perm], bt2, np.array(L, np.int32), k, lib=lib)
+    assert np.array_equal(out, base)
+
+
+def pin_verify_invalid_lengths(lib):
+    """Sequences with L < k+1, L beyond the table, or a page id outside the
+    cache yield NaN rows and are counted; valid ones are untouched."""
+    vi = workloads.make_verify([64, 64, 64, 64], 2, 2, 1, 8, seed=51, device="cpu")
+    qb, kb, vb = (workloads.bf16_bits(t) for t in (vi.q, vi.k_cache, vi.v_cache))
+    bt = vi.block_table.numpy().copy()
+    L = np.array([64, 2, 65, 64], np.int32)
+    bt[3, 0] = kb.shape[0]
+    out, n_bad = oracle.verify(qb, kb, vb, bt, L, 2, lib=lib)
+    assert n_bad == 3
+    assert np.all(np.isfinite(out[0])) and np.all(np.isnan(out[1:]))
+
+
+# --------------------------------------------------------------------------
+# draft pins
+# --------------------------------------------------------------------------
+def _draft_positions_closed_form(t, n_sink, window):
+    """Mean logical position over V(t), in closed form."""
+    S = n_sink + window
+    if t <= S:
+        return (t - 1) / 2.0
+    s = min(n_sink, t)
+    sink_sum = s * (s - 1) / 2.0
+    lo = t - window
+    win_sum = window * (lo + t - 1) / 2.0
+    return (sink_sum + win_sum) / (s + window)
+
+
+def pin_draft_uniform_logits_closed_form(lib):
+    """q = 0: the draft output is the mean over the visible set V(t); value at
+    logical position p carries p, so the mean is a closed form in t, n_sink
+    and window.  Runs on the logical form and on the packed ring."""
+    D, Hkv, Hq = 4, 2, 4
+    for (n_sink, window) in [(4, 8), (0, 5), (1, 64), (3, 1)]:
+        S = n_sink + window
+        ts = np.array([1, 2, n_sink + 1, S - 1 if S > 1 else 1, S, S + 1, 2 * S + 3, 200],
+                      dtype=np.int32)
+        ts = np.maximum(ts, 1)
+        B, T = len(ts), int(ts.max())
+        vals = np.zeros((B, Hkv, T, D), np.float32)
+        vals[..., 0] = np.arange(T)[None, None, :]
+        vals[..., 1] = np.arange(Hkv)[None, :, None]
+        vals[..., 3] = 1.0
+        Vl = _f32_to_bf16_bits(vals)
+        Kl = _f32_to_bf16_bits(np.ones((B, Hkv, T, D), np.float32))
+        q = np.zeros((B, Hq, D), np.uint16)
+        lo, nb = oracle.draft_logical(q, Kl, Vl, ts, n_sink, window, lib=lib)
+        ring = oracle.ring_pack(Kl, Vl, ts, n_sink, window, lib=lib)
+        ro, nb2 = oracle.draft_ring(q, ring, ts, n_sink, window, lib=lib)
+        assert nb == 0 and nb2 == 0
+        for b, t in enumerate(ts):
+            for h in range(Hq):
+                exp = np.array([_draft_positions_closed_form(int(t), n_sink, window),
+                                h // (Hq // Hkv), 0.0, 1.0])
+                np.testing.assert_allclose(lo[b, h], exp, rtol=0, atol=1e-12)
+                np.testing.assert_allclose(ro[b, h], exp, rtol=0, atol=1e-12)
+
+
+def pin_draft_matches_sdpa(lib):
+    """Logical form vs torch fp64 SDPA with the sink + window mask written as
+    a boolean mask over positions 0..T-1."""
+    rng = np.random.default_rng(61)
+    B, Hq, Hkv, D, T = 3, 4, 2, 16, 90
+    for (n_sink, window) in [(4, 16), (0, 7), (2, 100)]:
+        ts = np.array([1, 37, 90], np.int32)
+        Kf = rng.standard_normal((B, Hkv, T, D)).astype(np.float32)
+        Vf = rng.standard_normal((B, Hkv, T, D)).astype(np.float32)
+        Qf = (rng.standard_normal((B, Hq, D)) / 4).astype(np.float32)
+        Kb, Vb, Qb = (torch.from_numpy(x).to(torch.bfloat16) for x in (Kf, Vf, Qf))
+        bits = lambda t: t.view(torch.int16).numpy().view(np.uint16)
+        out, _ = oracle.draft_logical(bits(Qb), bits(Kb), bits(Vb), ts, n_sink, window, lib=lib)
+        G = Hq // Hkv
+        for b, t in enumerate(ts):
+            pos = torch.arange(T)
+            mask = (pos < t) & ((pos < n_sink) | (pos >= t - window))
+            K = Kb[b].double().repeat_interleave(G, 0)
+            V = Vb[b].double().repeat_interleave(G, 0)
+            Q = Qb[b].double()[:, None, :]
+            ref = torch.nn.functional.scaled_dot_product_attention(
+                Q, K, V, attn_mask=mask[None, None, :].expand(Hq, 1, T), scale=1.0)
+            np.testing.assert_allclose(out[b], ref[:, 0].numpy(), rtol=1e-12, atol=1e-12)
+
+
+def pin_draft_ring_equals_logical(lib):
+    """Packing a logical memory into the bounded cache and attending over the
+    ring equals attending over the logical memory with the mask, bit for bit."""
+    rng = np.random.default_rng(71)
+    B, Hq, Hkv, D = 4, 4, 1, 8
+    for (n_sink, window) in [(4, 16), (0, 9), (16, 1)]:
+        ts = np.array([3, 20, 21, 95], np.int32)
+        T = int(ts.max())
+        f = lambda *s: torch.from_numpy(rng.standard_normal(s).astype(np.float32)).to(torch.bfloat16)
+        bits = lambda t: t.view(torch.int16).numpy().view(np.uint16)
+        Kl, Vl, Q = bits(f(B, Hkv, T, D)), bits(f(B, Hkv, T, D)), bits(f(B, Hq, D))
+        lo, _ = oracle.draft_logical(Q, Kl, Vl, ts, n_sink, window, lib=lib)
+        ring = oracle.ring_pack(Kl, Vl, ts, n_sink, window, lib=lib)
+        ro, _ = oracle.draft_ring(Q, ring, ts, n_sink, window, lib=lib)
+        assert np.array_equal(lo, ro)
+
+
+def pin_draft_window_covers_context(lib):
+    """window >= t: the draft output equals full attention over all t entries,
+    i.e. the verification oracle at k = 0 over a contiguous cache."""
+    rng = np.random.default_rng(81)
+    B, Hq, Hkv, D = 3, 4, 2, 16
+    n_sink, window = 2, 200
+    ts = np.array([1, 64, 150], np.int32)
+    S = n_sink + window
+    kv = torch.from_numpy(rng.standard_normal((B, 2, Hkv, S, D)).astype(np.float32)).to(torch.bfloat16)
+    q = torch.from_numpy((rng.standard_normal((B, Hq, D)) / 4).astype(np.float32)).to(torch.bfloat16)
+    bits = lambda t: t.contiguous().view(torch.int16).numpy().view(np.uint16)
+    dr, _ = oracle.draft_ring(bits(q), bits(kv), ts, n_sink, window, lib=lib)
+    pages = (S + PAGE - 1) // PAGE
+    kc = torch.zeros((B * pages, Hkv, PAGE, D), dtype=torch.bfloat16)
+    vc = torch.zeros_like(kc)
+    for b in range(B):
+        for p in range(pages):
+            lo, hi = p * PAGE, min(S, (p + 1) * PAGE)
+            kc[b * pages + p, :, :hi - lo] = kv[b, 0, :, lo:hi]
+            vc[b * pages + p, :, :hi - lo] = kv[b, 1, :, lo:hi]
+    bt = np.arange(B * pages, dtype=np.int32).reshape(B, pages)
+    full, _ = oracle.verify(bits(q[:, None]), bits(kc), bits(vc), bt, ts, 0, lib=lib)
+    np.testing.assert_allclose(dr, full[:, 0], rtol=1e-15, atol=1e-15)
+
+
+def pin_draft_slot_is_bijective(lib):
+    """For every t >= S the visible positions fill each of the S slots exactly
+    once; sinks keep their own slot; entries p and p+window share a slot."""
+    for (n_sink, window) in [(0, 1), (1, 64), (16, 512), (4, 7)]:
+        S = n_sink + window
+        for t in [S, S + 1, 3 * S + 5]:
+            vis = [p for p in range(t) if p < n_sink or p >= t - window]
+            slots = sorted(oracle.draft_slot(p, n_sink, window, lib=lib) for p in vis)
+            assert slots == list(range(S))
+        for p in range(n_sink):
+            assert oracle.draft_slot(p, n_sink, window, lib=lib) == p
+        for p in range(n_sink, n_sink + 3 * window):
+            assert oracle.draft_slot(p, n_sink, window, lib=lib) == \
+                oracle.draft_slot(p + window, n_sink, window, lib=lib)
+            assert oracle.draft_slot(p, n_sink, window, lib=lib) >= n_sink
+
+
+def pin_draft_invalid_t(lib):
+    """t = 0 (no memory entry yet) yields NaN and is counted."""
+    di = workloads.make_draft([0, 5], 2, 1, 8, 1, 4, seed=3, device="cpu")
+    out, n_bad = oracle.draft_ring(workloads.bf16_bits(di.q), workloads.bf16_bits(di.kv),
+                                   di.ctx_lens.numpy(), 1, 4, lib=lib)
+    assert n_bad == 1 and np.all(np.isnan(out[0])) and np.all(np.isfinite(out[1]))
+
+
+ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -1,0 +1,72 @@
+"""Each plausible mistake planted in a copy of the oracle must trip a pin.
+
+The mutation is applied to a temporary copy of oracle/spire_oracle.c, which is
+compiled on the CPU; the real oracle is never modified.  A mutant that passes
+every pin would mean the pins cannot tell that mistake from the definition.
+"""
+import os
+import shutil
+import subprocess
+import tempfile
+
+import pytest
+
+import oracle
+import oracle_pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "spire_oracle.c")
+
+# (id, text in the oracle, replacement) -- one plausible mistake each.
+MUTATIONS = [
+    ("no_causal_offset", "int64_t n_i = L - c->k + i;", "int64_t n_i = L - c->k;"),
+    ("causal_off_by_one", "int64_t n_i = L - c->k + i;", "int64_t n_i = L - c->k + i + 1;"),
+    ("gqa_modulo", "int32_t g = h / group;", "int32_t g = h % c->Hkv;"),
+    ("page_index_no_table",
+     "int64_t page = c->block_table[(int64_t)b * c->max_pages + j / c->page_size];",
+     "int64_t page = (int64_t)b * c->max_pages + j / c->page_size;"),
+    ("page_slot_wrong", "int64_t slot = j % c->page_size;", "int64_t slot = j / c->page_size;"),
+    ("exp2_not_exp", "double p = exp(scores[j] - m);", "double p = exp2(scores[j] - m);"),
+    ("scale_dropped", "s *= scale;", "s *= 1.0;"),
+    ("no_normalise", "out[d] /= l;", "out[d] /= 1.0;"),
+    ("transposed_qk", "s += bf16_to_double(q[d]) * bf16_to_double(keys[j][d]);",
+     "s += bf16_to_double(q[d]) * bf16_to_double(vals[j][d]);"),
+    ("window_off_by_one", "return p < n_sink || p >= t - window;",
+     "return p < n_sink || p > t - window;"),
+    ("sinks_dropped", "return p < n_sink || p >= t - window;", "return p >= t - window;"),
+    ("window_one_extra", "return p < n_sink || p >= t - window;",
+     "return p < n_sink || p >= t - window - 1;"),
+    ("ring_no_sink_offset", "return n_sink + (p - n_sink) % window;",
+     "return (p - n_sink) % window;"),
+    ("ring_reads_k_as_v",
+     "vals[n] = base + ((((int64_t)b * 2 + 1) * c->Hkv + g) * S + s) * c->D;",
+     "vals[n] = base + ((((int64_t)b * 2 + 0) * c->Hkv + g) * S + s) * c->D;"),
+    ("query_row_stride", "const uint16_t *qi = c->q + (((int64_t)b * rows + i) * c->Hq + h) * c->D;",
+     "const uint16_t *qi = c->q + (((int64_t)b * rows) * c->Hq + h) * c->D;"),
+]
+
+
+@pytest.fixture(scope="module")
+def workdir():
+    d = tempfile.mkdtemp(prefix="spire_mutants_")
+    yield d
+    shutil.rmtree(d, ignore_errors=True)
+
+
+@pytest.mark.parametrize("mid,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_mutant_is_caught(mid, old, new, workdir):
+    text = open(SRC).read()
+    assert text.count(old) == 1, "mutation anchor must occur exactly once: %r" % old
+    src = os.path.join(workdir, mid + ".c")
+    so = os.path.join(workdir, mid + ".so")
+    with open(src, "w") as f:
+        f.write(text.replace(old, new))
+    subprocess.run(["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-pthread", "-o", so, src,
+                    "-lm"], check=True)
+    lib = oracle.load(so)
+    caught = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(lib)
+        except (AssertionError, ValueError):
+            caught.append(pin.__name__)
+    assert caught, "mutant %s passed every pin" % mid
