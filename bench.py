@@ -1,0 +1,411 @@
+"""Benchmark of one SPIRe speculation round's attention on GB300.
+
+A step is one pass of the whole hot path over one batch: the verification
+attention of the k+1 block tokens (split plan, split attention, LSE combine)
+plus the k draft sink + window attention steps of the round (draft step j sees
+t = L - k + j memory entries).  The default workload is the uniform long-
+context config: B=64, L=8192, k=4, 32 query / 8 KV heads, D=128, 64-token pages
+in a seeded random order, draft 16 sink + 512 window.  Inputs are seeded
+synthetic N(0,1) bf16 tensors resident in HBM.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
+                    [--impl spire|reference]
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle
+on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+METRIC = "speculation-round attention tokens/s and HBM GB/s vs 8 TB/s at B=64, k=4, 1 GB300"
+HBM_NOMINAL_GBS = 8000.0
+SPIRE_TAU_K4_L512 = 3.401   # SPIRe average generation length at L=512, k=4 (Table 1)
+
+
+# ------------------------------------------------------------------ helpers
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self, t0, t1):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        rows = []
+        for ts, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            rows.append((ts, parts))
+        inside = [r for ts, r in rows if t0 - 0.25 <= ts <= t1 + 0.25] or [r for _, r in rows]
+        sm = [float(r[1]) for r in inside if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in inside if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i in range(4)
+                          if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(inside), "reasons": reasons}
+
+
+def verify_bytes(L, k, Hq, Hkv, D):
+    """Algorithmic bytes of one verification call: every visible K/V byte once,
+    q in (bf16), out (fp32), the block-table entries read and ctx_lens."""
+    L = np.asarray(L, dtype=np.int64)
+    B = L.size
+    kv = int(L.sum()) * 4 * Hkv * D
+    qo = B * (k + 1) * Hq * D * (2 + 4)
+    meta = int(((L + 63) // 64).sum()) * 4 + 4 * B
+    return kv + qo + meta
+
+
+def draft_bytes(t, S, Hq, Hkv, D):
+    t = np.asarray(t, dtype=np.int64)
+    B = t.size
+    return int(np.minimum(t, S).sum()) * 4 * Hkv * D + B * Hq * D * 6 + 4 * B
+
+
+def verify_flops(L, k, Hq, D):
+    L = np.asarray(L, dtype=np.int64)
+    rows = sum(int((L - k + i).sum()) for i in range(k + 1))
+    return 4 * D * Hq * rows
+
+
+# ------------------------------------------------------------------ oracle arm
+def run_oracle_sample(cfg, n_seq, threads):
+    """Time the fp64 oracle on the first n_seq sequences of the workload:
+    the verification call plus the k draft steps.  Returns (seconds, tokens)."""
+    import oracle
+    L = wl.sample_ctx_lens(cfg)[:n_seq]
+    vi = wl.make_verify(L, cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim,
+                        seed=cfg.seed, device="cpu", shuffle=cfg.paged_shuffle)
+    qb, kb, vb = wl.bf16_bits(vi.q), wl.bf16_bits(vi.k_cache), wl.bf16_bits(vi.v_cache)
+    bt, cl = vi.block_table.numpy(), vi.ctx_lens.numpy()
+    drafts = []
+    for j in range(cfg.k):
+        di = wl.make_draft(wl.draft_ctx_for_step(L, cfg.k, j), cfg.num_q_heads,
+                           cfg.num_kv_heads, cfg.head_dim, cfg.n_sink, cfg.window,
+                           seed=cfg.seed + 17 * (j + 1), device="cpu")
+        drafts.append((wl.bf16_bits(di.q), wl.bf16_bits(di.kv), di.ctx_lens.numpy()))
+    t0 = time.perf_counter()
+    oracle.verify(qb, kb, vb, bt, cl, cfg.k, threads=threads)
+    for (q, kv, t) in drafts:
+        oracle.draft_ring(q, kv, t, cfg.n_sink, cfg.window, threads=threads)
+    dt = time.perf_counter() - t0
+    return dt, n_seq * (cfg.k + 1)
+
+
+def oracle_sample_size(cfg, target_s=15.0, threads=None):
+    """Sequences of the workload that keep the oracle leg near target_s."""
+    dt, _ = run_oracle_sample(cfg, 1, threads)
+    n = int(max(1, min(cfg.batch, math.floor(target_s / max(dt, 1e-3)))))
+    return n
+
+
+def reference_arm(args, cfg):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    threads = os.cpu_count() or 1
+    n_seq = oracle_sample_size(cfg, target_s=max(1.0, 20.0 / max(1, args.steps + args.warmup)),
+                               threads=threads)
+    for _ in range(args.warmup):
+        run_oracle_sample(cfg, n_seq, threads)
+    times = []
+    tokens = 0
+    for _ in range(args.steps):
+        dt, tok = run_oracle_sample(cfg, n_seq, threads)
+        times.append(dt)
+        tokens = tok
+    per_step = statistics.mean(times)
+    value = tokens / per_step
+    sample = ("first %d of %d sequences per step (verify + %d draft steps), fp64 C oracle"
+              % (n_seq, cfg.batch, cfg.k))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": per_step * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ spire arm
+def spire_arm(args, cfg):
+    import torch
+
+    import paper_2504_06419_gb300 as spire
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+
+    k, Hq, Hkv, D = cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+    L = wl.sample_ctx_lens(cfg)
+    vi = wl.make_verify(L, k, Hq, Hkv, D, seed=cfg.seed, device=dev, shuffle=cfg.paged_shuffle)
+    drafts = [wl.make_draft(wl.draft_ctx_for_step(L, k, j), Hq, Hkv, D, cfg.n_sink, cfg.window,
+                            seed=cfg.seed + 17 * (j + 1), device=dev) for j in range(k)]
+    S = cfg.n_sink + cfg.window
+    vdesc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+    ddesc = spire.draft_desc(drafts[0].q, drafts[0].kv)
+    ws_v = torch.empty(spire.spire_verify_workspace_bytes(vdesc, k), dtype=torch.uint8, device=dev)
+    ws_d = torch.empty(spire.spire_draft_workspace_bytes(ddesc, cfg.n_sink, cfg.window),
+                       dtype=torch.uint8, device=dev)
+    out_v = torch.empty(vi.q.shape, dtype=torch.float32, device=dev)
+    out_d = [torch.empty(d.q.shape, dtype=torch.float32, device=dev) for d in drafts]
+    sptr = stream.cuda_stream
+
+    def call_verify(q=vi.q, ctx=vi.ctx_lens, bt=vi.block_table, out=out_v):
+        st = spire.spire_verify_attention(q, vi.k_cache, vi.v_cache, bt, ctx, k, vdesc, out,
+                                          ws_v, ws_v.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_verify_attention")
+
+    def call_draft(j, q=None, ctx=None, out=None):
+        d = drafts[j]
+        st = spire.spire_draft_sparse_attention(q if q is not None else d.q, d.kv,
+                                                ctx if ctx is not None else d.ctx_lens,
+                                                cfg.n_sink, cfg.window, ddesc,
+                                                out if out is not None else out_d[j], ws_d,
+                                                ws_d.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_draft_sparse_attention")
+
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # 2x the 129 MB L2
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    # ---- device-resident timing: per-step and per-call CUDA events
+    for _ in range(args.warmup):
+        call_verify()
+        for j in range(k):
+            call_draft(j)
+    torch.cuda.synchronize(dev)
+    err = spire.spire_get_device_error(ws_v, stream)
+    if err:
+        raise RuntimeError("device error word %d after warm-up" % err)
+
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(k + 2)] for _ in range(args.steps)]
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    sampler.start()
+    time.sleep(0.6)
+    barrier()
+    t0 = time.time()
+    for s in range(args.steps):
+        flush.fill_(s & 0xff)          # L2 flush between steps, outside the events
+        e = ev[s]
+        e[0].record(stream)
+        call_verify()
+        e[1].record(stream)
+        for j in range(k):
+            call_draft(j)
+            e[2 + j].record(stream)
+    barrier()
+    t1 = time.time()
+    clocks = sampler.stop(t0, t1)
+    step_ms = [e[0].elapsed_time(e[-1]) for e in ev]
+    verify_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    draft_ms = [[e[1 + j].elapsed_time(e[2 + j]) for j in range(k)] for e in ev]
+    ms = statistics.mean(step_ms)
+    v_ms = statistics.mean(verify_ms)
+    d_ms = statistics.mean(sum(x) for x in draft_ms)
+    if dist is not None:
+        t = torch.tensor([ms, v_ms, d_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, v_ms, d_ms = (float(x) for x in t.tolist())
+
+    B = cfg.batch
+    tokens = B * (k + 1)
+    value = world * tokens / (ms * 1e-3)
+    vb = verify_bytes(L, k, Hq, Hkv, D)
+    db = sum(draft_bytes(wl.draft_ctx_for_step(L, k, j), S, Hq, Hkv, D) for j in range(k))
+    hbm_peak, peak_kind = peaks()
+    v_gbs = vb / (v_ms * 1e-3) / 1e9
+    d_gbs = db / (d_ms * 1e-3) / 1e9
+
+    # ---- end to end through the C ABI with host buffers
+    pin = lambda t: t.detach().cpu().pin_memory()
+    h_q, h_ctx, h_bt = pin(vi.q), pin(vi.ctx_lens), pin(vi.block_table)
+    h_dq = [pin(d.q) for d in drafts]
+    h_dctx = [pin(d.ctx_lens) for d in drafts]
+    h_out = torch.empty(out_v.shape, dtype=torch.float32).pin_memory()
+    h_dout = [torch.empty(o.shape, dtype=torch.float32).pin_memory() for o in out_d]
+    d_q, d_ctx, d_bt = torch.empty_like(vi.q), torch.empty_like(vi.ctx_lens), torch.empty_like(vi.block_table)
+    d_dq = [torch.empty_like(d.q) for d in drafts]
+    d_dctx = [torch.empty_like(d.ctx_lens) for d in drafts]
+    h2d = (h_q.numel() * 2 + h_ctx.numel() * 4 + h_bt.numel() * 4 +
+           sum(x.numel() * 2 for x in h_dq) + sum(x.numel() * 4 for x in h_dctx))
+    d2h = h_out.numel() * 4 + sum(x.numel() * 4 for x in h_dout)
+
+    def e2e_step():
+        d_q.copy_(h_q, non_blocking=True)
+        d_ctx.copy_(h_ctx, non_blocking=True)
+        d_bt.copy_(h_bt, non_blocking=True)
+        call_verify(q=d_q, ctx=d_ctx, bt=d_bt, out=out_v)
+        h_out.copy_(out_v, non_blocking=True)
+        for j in range(k):
+            d_dq[j].copy_(h_dq[j], non_blocking=True)
+            d_dctx[j].copy_(h_dctx[j], non_blocking=True)
+            call_draft(j, q=d_dq[j], ctx=d_dctx[j], out=out_d[j])
+            h_dout[j].copy_(out_d[j], non_blocking=True)
+
+    for _ in range(max(3, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    e2e_steps = max(1, min(args.steps, 200))
+    e2e_ms = []
+    for s in range(e2e_steps):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        e2e_step()
+        b.record(stream)
+        b.synchronize()          # the step's result is on the host
+        e2e_ms.append(a.elapsed_time(b))
+    e2e_val = world * tokens / (statistics.mean(e2e_ms) * 1e-3)
+
+    if rank != 0:
+        if dist is not None:
+            dist.barrier()
+            dist.destroy_process_group()
+        return 0
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        threads = os.cpu_count() or 1
+        n_seq = oracle_sample_size(cfg, target_s=15.0, threads=threads)
+        dt, tok = run_oracle_sample(cfg, n_seq, threads)
+        cpu = {"value": tok / dt, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+               "sample": "first %d of %d sequences, verify + %d draft steps, fp64 C oracle, "
+                         "%.1f s" % (n_seq, cfg.batch, k, dt)}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "%s: B=%d, L=%s, k=%d, %d/%d heads, D=%d, 64-token pages "
+                               "(shuffled=%s), draft %d sink + %d window"
+                               % (cfg.name, B, ("%d" % L[0]) if cfg.ctx_dist == "fixed" else
+                                  "%s[%d,%d] (sum %d)" % (cfg.ctx_dist, cfg.ctx_lo, cfg.ctx_hi,
+                                                          int(L.sum())),
+                                  k, Hq, Hkv, D, cfg.paged_shuffle, cfg.n_sink, cfg.window),
+                   "global_batch": B, "seq_len": int(L.max()), "parallelism": "replicas",
+                   "l2": "flushed between steps (256 MB write); verify KV %.2f GB > L2"
+                         % (vb / 1e9)},
+        "roofline": {"kernel": "spire_verify_attention (plan + split + combine)",
+                     "bound": "hbm", "achieved": v_gbs, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": v_gbs / hbm_peak, "peak_kind": peak_kind,
+                     "frac_of_8TBs": v_gbs / HBM_NOMINAL_GBS,
+                     "algorithmic_bytes": vb, "traffic": None},
+        "detail": {"verify_ms": v_ms, "draft_ms_total": d_ms, "verify_gbs": v_gbs,
+                   "draft_gbs": d_gbs, "draft_bytes_per_round": db,
+                   "verify_tokens_per_s": world * tokens / (v_ms * 1e-3),
+                   "draft_tokens_per_s": world * B * k / (d_ms * 1e-3),
+                   "verify_tflops": verify_flops(L, k, Hq, D) / (v_ms * 1e-3) / 1e12,
+                   "tau_weighted_tokens_per_s_context": world * B * SPIRE_TAU_K4_L512 / (ms * 1e-3)},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h)},
+        "gpu_launches": 3 * (k + 1) * args.steps,
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="uniform8k", choices=sorted(wl.CONFIGS))
+    ap.add_argument("--impl", default="spire", choices=["spire", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    cfg = wl.CONFIGS[args.config]
+    if args.impl == "reference":
+        return reference_arm(args, cfg)
+    return spire_arm(args, cfg)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

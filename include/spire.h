@@ -47,6 +47,12 @@
 extern "C" {
 #endif
 
+#if defined(__GNUC__)
+#define SPIRE_API __attribute__((visibility("default")))
+#else
+#define SPIRE_API
+#endif
+
 /* Status of a host call. */
 typedef enum spire_status {
     SPIRE_OK = 0,
@@ -83,7 +89,7 @@ typedef struct spire_attn_desc {
  * Depends only on the shapes (batch, heads, head_dim) and k, not on the
  * device or on ctx_lens.  Returns 0 if desc is NULL or k < 0.
  */
-size_t spire_verify_workspace_bytes(const spire_attn_desc *desc, int32_t k);
+SPIRE_API size_t spire_verify_workspace_bytes(const spire_attn_desc *desc, int32_t k);
 
 /*
  * spire_verify_attention -- verification attention of one speculation round
@@ -113,7 +119,7 @@ size_t spire_verify_workspace_bytes(const spire_attn_desc *desc, int32_t k);
  *                share a workspace must be ordered (same stream).
  * Returns SPIRE_OK once the work is enqueued.
  */
-spire_status spire_verify_attention(const void *q, const void *k_cache,
+SPIRE_API spire_status spire_verify_attention(const void *q, const void *k_cache,
                                     const void *v_cache,
                                     const int32_t *block_table,
                                     const int32_t *ctx_lens, int32_t k,
@@ -125,7 +131,7 @@ spire_status spire_verify_attention(const void *q, const void *k_cache,
  * spire_draft_workspace_bytes -- workspace size for
  * spire_draft_sparse_attention.  Returns 0 for invalid arguments.
  */
-size_t spire_draft_workspace_bytes(const spire_attn_desc *desc, int32_t n_sink,
+SPIRE_API size_t spire_draft_workspace_bytes(const spire_attn_desc *desc, int32_t n_sink,
                                    int32_t window);
 
 /*
@@ -150,7 +156,7 @@ size_t spire_draft_workspace_bytes(const spire_attn_desc *desc, int32_t n_sink,
  *   workspace >= spire_draft_workspace_bytes(desc, n_sink, window) bytes.
  * desc->page_size / max_pages_per_seq / num_pages are ignored.
  */
-spire_status spire_draft_sparse_attention(const void *q, const void *kv,
+SPIRE_API spire_status spire_draft_sparse_attention(const void *q, const void *kv,
                                           const int32_t *ctx_lens,
                                           int32_t n_sink, int32_t window,
                                           const spire_attn_desc *desc,
@@ -162,18 +168,18 @@ spire_status spire_draft_sparse_attention(const void *q, const void *kv,
  * draft cache: p if p < n_sink, else n_sink + (p - n_sink) mod window.
  * Returns -1 for p < 0, n_sink < 0 or window < 1.  Host function.
  */
-int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
+SPIRE_API int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
 
 /*
  * spire_get_device_error -- copy the device error word of the most recent
  * call that used `workspace` into *code_out (0 = no error, else an OR of
  * SPIRE_DEVERR_* bits).  Synchronises `stream`.
  */
-spire_status spire_get_device_error(const void *workspace, int32_t *code_out,
+SPIRE_API spire_status spire_get_device_error(const void *workspace, int32_t *code_out,
                                     void *stream);
 
 /* spire_status_string -- static, human-readable name of a status. */
-const char *spire_status_string(spire_status status);
+SPIRE_API const char *spire_status_string(spire_status status);
 
 #ifdef __cplusplus
 }

@@ -1,0 +1,280 @@
+// spire_abi.cu -- the C ABI of libspire (declared in include/spire.h): host
+// validation, workspace layout, TMA descriptors and the launch sequence
+// plan -> split -> combine on the caller's stream.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include "spire.h"
+#include "spire_aux.cuh"
+#include "spire_launch.h"
+
+namespace spire {
+namespace {
+
+constexpr size_t kHeaderBytes = 256;
+constexpr double kLog2e = 1.4426950408889634;  // log2(e): softmax runs in base 2
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct WsLayout {
+    size_t seq_info, items, part_lse, part_o, total;
+};
+
+// Work-list bound: with chunk >= ceil(W / kTargetItems), the number of
+// items sum_{b,g} ceil(tiles_b / chunk) is at most kTargetItems + B * Hkv.
+WsLayout ws_layout(long long B, long long Hkv, long long R, long long D) {
+    const long long max_items = kTargetItems + B * Hkv;
+    WsLayout w{};
+    size_t off = kHeaderBytes;
+    w.seq_info = off; off += align256(size_t(B) * 16);
+    w.items = off;    off += align256(size_t(max_items) * 16);
+    w.part_lse = off; off += align256(size_t(max_items * R) * 4);
+    w.part_o = off;   off += align256(size_t(max_items * R * D) * 4);
+    w.total = off;
+    return w;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+spire_status check_common(const spire_attn_desc* d) {
+    if (!d) return SPIRE_ERR_INVALID_ARG;
+    if (d->batch < 0 || d->num_q_heads < 1 || d->num_kv_heads < 1) return SPIRE_ERR_INVALID_ARG;
+    if (d->num_q_heads % d->num_kv_heads != 0) return SPIRE_ERR_INVALID_ARG;
+    if (!std::isfinite(d->softmax_scale) || !(d->softmax_scale > 0.f)) return SPIRE_ERR_INVALID_ARG;
+    if (d->head_dim != 64 && d->head_dim != 128) return SPIRE_ERR_UNSUPPORTED;
+    return SPIRE_OK;
+}
+
+int rows_per_kv_head(const spire_attn_desc* d, int kp1) {
+    return (d->num_q_heads / d->num_kv_heads) * kp1;
+}
+
+// --------------------------------------------------------------- driver API
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 3-D bf16 view {D, rows, planes} read in 64 x 64 boxes with 128-byte swizzle.
+bool encode_kv_map(CUtensorMap* map, const void* base, uint64_t D, uint64_t rows,
+                   uint64_t planes) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {D, rows, planes};
+    cuuint64_t strides[2] = {D * 2, D * 2 * rows};
+    cuuint32_t box[3] = {64, 64, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+struct DeviceInfo {
+    int sms = 0;
+    int smem_optin = 0;
+};
+
+spire_status device_info(DeviceInfo* out) {
+    static std::mutex mu;
+    static DeviceInfo cache[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SPIRE_ERR_CUDA;
+    if (dev >= 0 && dev < 64) {
+        std::lock_guard<std::mutex> g(mu);
+        if (cache[dev].sms == 0) {
+            if (cudaDeviceGetAttribute(&cache[dev].sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+                cudaDeviceGetAttribute(&cache[dev].smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin,
+                                       dev) != cudaSuccess) {
+                cache[dev].sms = 0;
+                return SPIRE_ERR_CUDA;
+            }
+        }
+        *out = cache[dev];
+        return SPIRE_OK;
+    }
+    if (cudaDeviceGetAttribute(&out->sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&out->smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess)
+        return SPIRE_ERR_CUDA;
+    return SPIRE_OK;
+}
+
+// Shared launch sequence for both calls.
+spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorMap& tv,
+                 const int32_t* block_table, const int32_t* ctx_lens, int kp1,
+                 const spire_attn_desc* d, int cap, float* out, void* workspace,
+                 cudaStream_t stream) {
+    DeviceInfo di;
+    spire_status st = device_info(&di);
+    if (st != SPIRE_OK) return st;
+    if (di.smem_optin < kMaxDynSmem) return SPIRE_ERR_UNSUPPORTED;
+    const int B = d->batch, Hkv = d->num_kv_heads, D = d->head_dim;
+    const int R = rows_per_kv_head(d, kp1);
+    const WsLayout w = ws_layout(B, Hkv, R, D);
+    char* ws = static_cast<char*>(workspace);
+    int32_t* header = reinterpret_cast<int32_t*>(ws);
+    int4* seq_info = reinterpret_cast<int4*>(ws + w.seq_info);
+    int4* items = reinterpret_cast<int4*>(ws + w.items);
+    float* part_lse = reinterpret_cast<float*>(ws + w.part_lse);
+    float* part_o = reinterpret_cast<float*>(ws + w.part_o);
+
+    PlanParams pp{ctx_lens, seq_info, items, header, B, Hkv, kp1, mode,
+                  mode == kModeVerify ? d->max_pages_per_seq : 0, cap};
+    plan_kernel<<<1, kPlanThreads, 0, stream>>>(pp);
+    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+
+    SplitParams sp{};
+    sp.q = static_cast<const __nv_bfloat16*>(q);
+    sp.out = out;
+    sp.block_table = block_table;
+    sp.seq_info = seq_info;
+    sp.items = items;
+    sp.header = header;
+    sp.part_o = part_o;
+    sp.part_lse = part_lse;
+    sp.B = B;
+    sp.Hq = d->num_q_heads;
+    sp.Hkv = Hkv;
+    sp.G = d->num_q_heads / Hkv;
+    sp.kp1 = kp1;
+    sp.R = R;
+    sp.max_pages = mode == kModeVerify ? d->max_pages_per_seq : 0;
+    sp.num_pages = mode == kModeVerify ? d->num_pages : 0;
+    sp.mode = mode;
+    sp.sl2 = static_cast<float>(static_cast<double>(d->softmax_scale) * kLog2e);
+    const int mt = (R + 15) / 16;
+    cudaError_t e = D == 128 ? launch_split_d128(mt, tk, tv, sp, di.sms, stream)
+                             : launch_split_d64(mt, tk, tv, sp, di.sms, stream);
+    if (e != cudaSuccess) return SPIRE_ERR_CUDA;
+
+    CombineParams cp{seq_info, part_o, part_lse, out, B, d->num_q_heads, Hkv, sp.G, kp1, R, D};
+    combine_kernel<<<B * Hkv, 256, 0, stream>>>(cp);
+    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+    return SPIRE_OK;
+}
+
+}  // namespace
+}  // namespace spire
+
+using namespace spire;
+
+extern "C" {
+
+size_t spire_verify_workspace_bytes(const spire_attn_desc* desc, int32_t k) {
+    if (check_common(desc) != SPIRE_OK || k < 0 || k >= SPIRE_MAX_ROWS_PER_KV_HEAD) return 0;
+    const int R = rows_per_kv_head(desc, k + 1);
+    return ws_layout(desc->batch, desc->num_kv_heads, R, desc->head_dim).total;
+}
+
+size_t spire_draft_workspace_bytes(const spire_attn_desc* desc, int32_t n_sink, int32_t window) {
+    if (check_common(desc) != SPIRE_OK || n_sink < 0 || window < 1) return 0;
+    const int R = rows_per_kv_head(desc, 1);
+    return ws_layout(desc->batch, desc->num_kv_heads, R, desc->head_dim).total;
+}
+
+spire_status spire_verify_attention(const void* q, const void* k_cache, const void* v_cache,
+                                    const int32_t* block_table, const int32_t* ctx_lens,
+                                    int32_t k, const spire_attn_desc* desc, float* out,
+                                    void* workspace, size_t ws_bytes, void* stream) {
+    spire_status st = check_common(desc);
+    if (st != SPIRE_OK) return st;
+    if (k < 0) return SPIRE_ERR_INVALID_ARG;
+    if (desc->page_size != kPage) return SPIRE_ERR_UNSUPPORTED;
+    if (desc->max_pages_per_seq < 1 || desc->num_pages < 1) return SPIRE_ERR_INVALID_ARG;
+    if (rows_per_kv_head(desc, 1) > SPIRE_MAX_ROWS_PER_KV_HEAD ||
+        (long long)rows_per_kv_head(desc, 1) * (k + 1LL) > SPIRE_MAX_ROWS_PER_KV_HEAD)
+        return SPIRE_ERR_UNSUPPORTED;
+    // TMA plane index page * Hkv + g and the block-table offset are int32
+    if ((long long)desc->num_pages * desc->num_kv_heads >= (1LL << 31) ||
+        (long long)desc->batch * desc->max_pages_per_seq >= (1LL << 31) ||
+        (long long)desc->max_pages_per_seq * kPage >= (1LL << 31))
+        return SPIRE_ERR_UNSUPPORTED;
+    if (desc->batch == 0) return SPIRE_OK;
+    if (!q || !k_cache || !v_cache || !block_table || !ctx_lens || !out)
+        return SPIRE_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+        !aligned(block_table, 4) || !aligned(ctx_lens, 4))
+        return SPIRE_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || ws_bytes < spire_verify_workspace_bytes(desc, k))
+        return SPIRE_ERR_WORKSPACE;
+
+    CUtensorMap tk, tv;
+    const uint64_t planes = uint64_t(desc->num_pages) * uint64_t(desc->num_kv_heads);
+    if (!encode_kv_map(&tk, k_cache, desc->head_dim, kPage, planes) ||
+        !encode_kv_map(&tv, v_cache, desc->head_dim, kPage, planes))
+        return SPIRE_ERR_CUDA;
+    return run(kModeVerify, q, tk, tv, block_table, ctx_lens, k + 1, desc, 0, out, workspace,
+               static_cast<cudaStream_t>(stream));
+}
+
+spire_status spire_draft_sparse_attention(const void* q, const void* kv, const int32_t* ctx_lens,
+                                          int32_t n_sink, int32_t window,
+                                          const spire_attn_desc* desc, float* out,
+                                          void* workspace, size_t ws_bytes, void* stream) {
+    spire_status st = check_common(desc);
+    if (st != SPIRE_OK) return st;
+    if (n_sink < 0 || window < 1) return SPIRE_ERR_INVALID_ARG;
+    const long long S = (long long)n_sink + window;
+    if (S > (1LL << 30)) return SPIRE_ERR_UNSUPPORTED;
+    if (rows_per_kv_head(desc, 1) > SPIRE_MAX_ROWS_PER_KV_HEAD) return SPIRE_ERR_UNSUPPORTED;
+    if ((long long)desc->batch * 2 * desc->num_kv_heads >= (1LL << 31)) return SPIRE_ERR_UNSUPPORTED;
+    if (desc->batch == 0) return SPIRE_OK;
+    if (!q || !kv || !ctx_lens || !out) return SPIRE_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(kv, 16) || !aligned(out, 16) || !aligned(ctx_lens, 4))
+        return SPIRE_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) ||
+        ws_bytes < spire_draft_workspace_bytes(desc, n_sink, window))
+        return SPIRE_ERR_WORKSPACE;
+
+    CUtensorMap tkv;
+    const uint64_t planes = uint64_t(desc->batch) * 2u * uint64_t(desc->num_kv_heads);
+    if (!encode_kv_map(&tkv, kv, desc->head_dim, uint64_t(S), planes)) return SPIRE_ERR_CUDA;
+    return run(kModeDraft, q, tkv, tkv, nullptr, ctx_lens, 1, desc, int(S), out, workspace,
+               static_cast<cudaStream_t>(stream));
+}
+
+int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {
+    if (pos < 0 || n_sink < 0 || window < 1) return -1;
+    if (pos < n_sink) return pos;
+    return n_sink + (pos - n_sink) % window;
+}
+
+spire_status spire_get_device_error(const void* workspace, int32_t* code_out, void* stream) {
+    if (!workspace || !code_out) return SPIRE_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return SPIRE_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return SPIRE_ERR_CUDA;
+    *code_out = v;
+    return SPIRE_OK;
+}
+
+const char* spire_status_string(spire_status status) {
+    switch (status) {
+        case SPIRE_OK: return "SPIRE_OK";
+        case SPIRE_ERR_INVALID_ARG: return "SPIRE_ERR_INVALID_ARG";
+        case SPIRE_ERR_UNSUPPORTED: return "SPIRE_ERR_UNSUPPORTED";
+        case SPIRE_ERR_WORKSPACE: return "SPIRE_ERR_WORKSPACE";
+        case SPIRE_ERR_CUDA: return "SPIRE_ERR_CUDA";
+    }
+    return "SPIRE_ERR_UNKNOWN";
+}
+
+}  // extern "C"

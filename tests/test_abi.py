@@ -1,0 +1,122 @@
+"""The C ABI without a GPU: the library loads, exports every function that
+include/spire.h declares, and rejects bad host arguments before launching."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "spire.h")
+
+
+@pytest.fixture(scope="module")
+def spire():
+    import __graft_entry__
+    __graft_entry__._load_build_module().build()
+    import paper_2504_06419_gb300 as m
+    return m
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"SPIRE_API\s+[\w\s\*]+?\b(spire_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    assert names == sorted([
+        "spire_verify_workspace_bytes", "spire_verify_attention",
+        "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
+        "spire_get_device_error", "spire_status_string"]), names
+
+
+def test_library_exports_every_declared_symbol(spire):
+    lib = ctypes.CDLL(spire._lib.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(spire._lib.EXPORTED) == set(declared_functions())
+
+
+def test_status_strings(spire):
+    assert spire.spire_status_string(0) == "SPIRE_OK"
+    assert spire.spire_status_string(3) == "SPIRE_ERR_WORKSPACE"
+    assert spire.spire_status_string(99) == "SPIRE_ERR_UNKNOWN"
+
+
+def test_draft_slot_host(spire):
+    assert spire.spire_draft_slot(3, 4, 64) == 3
+    assert spire.spire_draft_slot(4, 4, 64) == 4
+    assert spire.spire_draft_slot(68, 4, 64) == 4
+    assert spire.spire_draft_slot(69, 4, 64) == 5
+    assert spire.spire_draft_slot(-1, 4, 64) == -1
+    assert spire.spire_draft_slot(5, 4, 0) == -1
+
+
+def _desc(spire, **kw):
+    d = dict(batch=2, num_q_heads=8, num_kv_heads=2, head_dim=128, page_size=64,
+             max_pages_per_seq=4, num_pages=8, softmax_scale=1.0)
+    d.update(kw)
+    return spire.make_desc(**d)
+
+
+FAKE = 1 << 20   # a 16-byte aligned non-null "device" address; never dereferenced here
+
+
+def _verify(spire, desc, k=4, ws_bytes=None, **ptrs):
+    p = dict(q=FAKE, kc=FAKE, vc=FAKE, bt=FAKE, cl=FAKE, out=FAKE, ws=FAKE)
+    p.update(ptrs)
+    if ws_bytes is None:
+        ws_bytes = spire.spire_verify_workspace_bytes(desc, k)
+    return spire.spire_verify_attention(p["q"], p["kc"], p["vc"], p["bt"], p["cl"], k, desc,
+                                        p["out"], p["ws"], ws_bytes, 0)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(num_q_heads=7), 1),          # Hq % Hkv != 0
+    (dict(num_kv_heads=0), 1),
+    (dict(batch=-1), 1),
+    (dict(head_dim=96), 2),            # unsupported head_dim
+    (dict(page_size=32), 2),           # unsupported page size
+    (dict(softmax_scale=0.0), 1),
+    (dict(softmax_scale=float("nan")), 1),
+    (dict(max_pages_per_seq=0), 1),
+])
+def test_verify_rejects_bad_desc(spire, kw, code):
+    assert _verify(spire, _desc(spire, **kw), ws_bytes=1 << 30) == code
+
+
+def test_verify_rejects_bad_args(spire):
+    d = _desc(spire)
+    assert _verify(spire, d, k=-1, ws_bytes=1 << 30) == 1
+    assert _verify(spire, d, k=32, ws_bytes=1 << 30) == 2          # 4 * 33 > 128 rows
+    assert _verify(spire, d, q=0) == 1
+    assert _verify(spire, d, out=0) == 1
+    assert _verify(spire, d, q=FAKE + 2) == 1                      # misaligned
+    assert _verify(spire, d, ws=0) == 3
+    assert _verify(spire, d, ws=FAKE + 16) == 3                    # workspace misaligned
+    assert _verify(spire, d, ws_bytes=spire.spire_verify_workspace_bytes(d, 4) - 1) == 3
+    assert _verify(spire, _desc(spire, batch=0), q=0, kc=0, ws=0, ws_bytes=0) == 0
+
+
+def test_draft_rejects_bad_args(spire):
+    d = _desc(spire)
+    ws = spire.spire_draft_workspace_bytes(d, 4, 64)
+    f = spire.spire_draft_sparse_attention
+    assert f(FAKE, FAKE, FAKE, -1, 64, d, FAKE, FAKE, ws, 0) == 1
+    assert f(FAKE, FAKE, FAKE, 4, 0, d, FAKE, FAKE, ws, 0) == 1
+    assert f(0, FAKE, FAKE, 4, 64, d, FAKE, FAKE, ws, 0) == 1
+    assert f(FAKE, FAKE, FAKE, 4, 64, d, FAKE, FAKE, ws - 1, 0) == 3
+    assert f(FAKE, FAKE, FAKE, 4, 64, _desc(spire, head_dim=80), FAKE, FAKE, ws, 0) == 2
+    assert spire.spire_draft_workspace_bytes(d, 4, 0) == 0
+
+
+def test_workspace_sizes_depend_only_on_shapes(spire):
+    d = _desc(spire, batch=64, num_q_heads=32, num_kv_heads=8)
+    a = spire.spire_verify_workspace_bytes(d, 4)
+    assert a > 0 and a % 256 == 0
+    assert spire.spire_verify_workspace_bytes(d, 8) > a
+    assert spire.spire_verify_workspace_bytes(_desc(spire, batch=64, num_q_heads=32,
+                                                    num_kv_heads=8, num_pages=10 ** 6), 4) == a
+    assert spire.spire_draft_workspace_bytes(d, 16, 512) == spire.spire_draft_workspace_bytes(d, 0, 9)
+    assert spire.spire_verify_workspace_bytes(None, 4) == 0

@@ -1,0 +1,77 @@
+"""Full-size parity on the benchmark workloads.
+
+Each call runs at full size in the same launch configuration the benchmark
+times; the oracle then recomputes a seeded sample of sequences (always
+including the shortest and the longest) over every head and block row, and
+the sampled outputs must match within max-abs 1e-2 and relative L2 1e-3.
+"""
+import numpy as np
+import pytest
+import torch
+
+import parity
+import workloads as wl
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def spire():
+    import paper_2504_06419_gb300 as m
+    return m
+
+
+def _sample(L, n, seed):
+    rng = np.random.default_rng(seed)
+    pick = set(rng.choice(len(L), size=min(n, len(L)), replace=False).tolist())
+    pick.add(int(np.argmin(L)))
+    pick.add(int(np.argmax(L)))
+    return sorted(pick)
+
+
+@pytest.mark.parametrize("name", ["tiny", "uniform8k", "ragged", "big"])
+def test_verify_full_config(spire, name):
+    cfg = wl.CONFIGS[name]
+    L = wl.sample_ctx_lens(cfg)
+    vi = wl.make_verify(L, cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim,
+                        seed=cfg.seed, device=DEV, shuffle=cfg.paged_shuffle)
+    desc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+    ws = torch.empty(spire.spire_verify_workspace_bytes(desc, cfg.k), dtype=torch.uint8,
+                     device=DEV)
+    out = spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens,
+                                 cfg.k, workspace=ws)
+    assert spire.spire_get_device_error(ws) == 0
+    seqs = _sample(L, 4, cfg.seed)
+    sub = parity.compact_verify(vi, seqs)
+    ref, n_bad = parity.oracle_verify(sub)
+    assert n_bad == 0
+    got = out[torch.tensor(seqs, device=DEV)].cpu().numpy()
+    parity.assert_close(got, ref, "verify %s sequences %s" % (name, seqs))
+    del vi, out, ws
+    torch.cuda.empty_cache()
+
+
+DRAFT_RUNS = [("tiny", None), ("uniform8k", None), ("ragged", None), ("big", None),
+              ("draft_sweep", 256), ("draft_sweep", 1024), ("draft_sweep", 4096)]
+
+
+@pytest.mark.parametrize("name,window", DRAFT_RUNS, ids=["%s-%s" % r for r in DRAFT_RUNS])
+def test_draft_full_config(spire, name, window):
+    cfg = wl.CONFIGS[name]
+    w = window or cfg.window
+    L = wl.sample_ctx_lens(cfg)
+    for j in (0, cfg.k - 1):
+        t = wl.draft_ctx_for_step(L, cfg.k, j)
+        di = wl.make_draft(t, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim, cfg.n_sink, w,
+                           seed=cfg.seed + 17 * (j + 1), device=DEV)
+        out = parity.gpu_draft(spire, di)
+        seqs = _sample(t, 8, cfg.seed + j)
+        sel = torch.tensor(seqs, device=DEV)
+        sub = wl.DraftInputs(q=di.q[sel].contiguous(), kv=di.kv[sel].contiguous(),
+                             ctx_lens=di.ctx_lens[sel].contiguous(), n_sink=cfg.n_sink, window=w)
+        ref, n_bad = parity.oracle_draft(sub)
+        assert n_bad == 0
+        parity.assert_close(out[sel].cpu().numpy(), ref, "draft %s w=%d step %d" % (name, w, j))
+        del di, out
+    torch.cuda.empty_cache()

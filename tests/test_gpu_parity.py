@@ -1,0 +1,220 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the fp64
+oracle on the same seeded inputs, plus the exactness properties of indexing."""
+import numpy as np
+import pytest
+import torch
+
+import parity
+import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def spire():
+    import paper_2504_06419_gb300 as m
+    return m
+
+
+DEV = "cuda"
+
+
+# ---------------------------------------------------------------- verify
+VERIFY_CASES = [
+    # (ctx_lens, k, Hq, Hkv, D)
+    ([256, 300], 4, 4, 1, 64),                 # the tiny config's shapes
+    ([5, 63, 64, 65, 129], 4, 32, 8, 128),    # ragged tails around the tile size
+    ([1, 2, 3, 64], 0, 8, 8, 128),             # G = 1, k = 0 (plain decoding), L = 1
+    ([9, 10, 200], 8, 64, 8, 128),             # G = 8, k = 8: 72 rows per KV head
+    ([2, 3000, 777], 1, 16, 2, 64),            # several splits, D = 64
+    ([4100, 70, 1000, 2049], 4, 32, 8, 128),   # splits + ragged
+    ([17, 33], 15, 8, 1, 128),                 # 128 rows per KV head (maximum)
+    ([100, 260], 2, 6, 2, 128),                # G = 3 (rows not a multiple of 8)
+]
+
+
+@pytest.mark.parametrize("case", VERIFY_CASES, ids=[str(i) for i in range(len(VERIFY_CASES))])
+def test_verify_matches_oracle(spire, case):
+    L, k, Hq, Hkv, D = case
+    vi = wl.make_verify(L, k, Hq, Hkv, D, seed=100 + len(L), device=DEV, poison=True,
+                        spare_pages=3)
+    desc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+    ws = torch.empty(spire.spire_verify_workspace_bytes(desc, k), dtype=torch.uint8, device=DEV)
+    got = spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, k,
+                                 workspace=ws)
+    assert spire.spire_get_device_error(ws) == 0
+    ref, n_bad = parity.oracle_verify(vi)
+    assert n_bad == 0
+    parity.assert_close(got.cpu().numpy(), ref, "verify %s" % (case,))
+
+
+def test_verify_tiny_config(spire):
+    cfg = wl.CONFIGS["tiny"]
+    vi = wl.make_verify(wl.sample_ctx_lens(cfg), cfg.k, cfg.num_q_heads, cfg.num_kv_heads,
+                        cfg.head_dim, seed=cfg.seed, device=DEV, shuffle=False, poison=True)
+    got = parity.gpu_verify(spire, vi).cpu().numpy()
+    ref, _ = parity.oracle_verify(vi)
+    parity.assert_close(got, ref, "tiny verify")
+
+
+def test_verify_scale(spire):
+    vi = wl.make_verify([130, 64], 2, 8, 2, 128, seed=7, device=DEV, q_std=1.0)
+    vi.scale = 0.088388
+    got = parity.gpu_verify(spire, vi).cpu().numpy()
+    ref, _ = parity.oracle_verify(vi)
+    parity.assert_close(got, ref, "scaled verify")
+
+
+def test_verify_page_permutation_bit_exact(spire):
+    L = [700, 64, 129]
+    a = wl.make_verify(L, 4, 32, 8, 128, seed=9, device=DEV, shuffle=False)
+    out_a = parity.gpu_verify(spire, a)
+    perm = torch.randperm(a.k_cache.shape[0], generator=torch.Generator().manual_seed(1)).to(DEV)
+    inv = torch.argsort(perm)
+    bt = torch.where(a.block_table >= 0, inv[a.block_table.clamp(min=0).long()].int(),
+                     a.block_table)
+    b = wl.VerifyInputs(q=a.q, k_cache=a.k_cache[perm].contiguous(),
+                        v_cache=a.v_cache[perm].contiguous(), block_table=bt,
+                        ctx_lens=a.ctx_lens, k=a.k)
+    out_b = parity.gpu_verify(spire, b)
+    assert torch.equal(out_a, out_b)
+
+
+def test_verify_nan_poison_bit_exact_and_deterministic(spire):
+    L = [1000, 65, 5, 5000]
+    clean = wl.make_verify(L, 4, 32, 8, 128, seed=11, device=DEV, poison=False, spare_pages=2)
+    pois = wl.make_verify(L, 4, 32, 8, 128, seed=11, device=DEV, poison=True, spare_pages=2)
+    o1 = parity.gpu_verify(spire, clean)
+    o2 = parity.gpu_verify(spire, pois)
+    o3 = parity.gpu_verify(spire, pois)
+    assert torch.isfinite(o2).all()
+    assert torch.equal(o1, o2)
+    assert torch.equal(o2, o3)
+
+
+def test_verify_causality_bit_exact(spire):
+    L, k = [777, 64], 4
+    vi = wl.make_verify(L, k, 32, 8, 128, seed=13, device=DEV)
+    base = parity.gpu_verify(spire, vi)
+    for i in range(1, k + 1):
+        kc, vc = vi.k_cache.clone(), vi.v_cache.clone()
+        for b, Lb in enumerate(L):
+            j = Lb - k + i - 1
+            page = int(vi.block_table[b, j // 64])
+            kc[page, :, j % 64] = 3.0
+            vc[page, :, j % 64] = 100.0
+        vj = wl.VerifyInputs(q=vi.q, k_cache=kc, v_cache=vc, block_table=vi.block_table,
+                             ctx_lens=vi.ctx_lens, k=k)
+        out = parity.gpu_verify(spire, vj)
+        assert torch.equal(out[:, :i], base[:, :i])
+        assert not torch.allclose(out[:, i], base[:, i])
+
+
+def test_verify_row_equals_decode(spire):
+    L, k = [900, 130, 64], 4
+    vi = wl.make_verify(L, k, 32, 8, 128, seed=17, device=DEV)
+    out = parity.gpu_verify(spire, vi).cpu().numpy()
+    for i in range(k + 1):
+        di = wl.VerifyInputs(q=vi.q[:, i:i + 1].contiguous(), k_cache=vi.k_cache,
+                             v_cache=vi.v_cache, block_table=vi.block_table,
+                             ctx_lens=(vi.ctx_lens - k + i).contiguous(), k=0)
+        dec = parity.gpu_verify(spire, di).cpu().numpy()
+        rel, mx = parity.errors(out[:, i], dec[:, 0])
+        assert rel <= 1e-5 and mx <= 1e-5, (i, rel, mx)
+
+
+def test_verify_constant_v(spire):
+    vi = wl.make_verify([300, 5000], 4, 32, 8, 128, seed=19, device=DEV)
+    vi.v_cache.fill_(0.8125)
+    out = parity.gpu_verify(spire, vi)
+    assert torch.allclose(out, torch.full_like(out, 0.8125), rtol=0, atol=1e-6)
+
+
+def test_verify_device_errors(spire):
+    L = [200, 200, 200, 200]
+    vi = wl.make_verify(L, 4, 8, 2, 128, seed=23, device=DEV)
+    ctx = torch.tensor([200, 3, 200, 10 ** 6], dtype=torch.int32, device=DEV)  # too short / too long
+    bt = vi.block_table.clone()
+    bt[2, 1] = vi.k_cache.shape[0] + 5                                         # page outside cache
+    v2 = wl.VerifyInputs(q=vi.q, k_cache=vi.k_cache, v_cache=vi.v_cache, block_table=bt,
+                         ctx_lens=ctx, k=4)
+    desc = spire.verify_desc(v2.q, v2.k_cache, v2.block_table)
+    ws = torch.empty(spire.spire_verify_workspace_bytes(desc, 4), dtype=torch.uint8, device=DEV)
+    out = spire.verify_attention(v2.q, v2.k_cache, v2.v_cache, v2.block_table, v2.ctx_lens, 4,
+                                 workspace=ws)
+    err = spire.spire_get_device_error(ws)
+    assert err == 3, err                   # CTX_LEN | PAGE_ID
+    assert torch.isnan(out[1:]).all()
+    ref, _ = parity.oracle_verify(vi)
+    parity.assert_close(out[0].cpu().numpy(), ref[0], "valid row beside bad ones")
+    # a clean call on the same workspace clears the word
+    spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, 4,
+                           workspace=ws)
+    assert spire.spire_get_device_error(ws) == 0
+
+
+def test_verify_empty_batch(spire):
+    desc = spire.make_desc(0, 8, 2, 128, 64, 4, 4)
+    assert spire.spire_verify_attention(0, 0, 0, 0, 0, 4, desc, 0, 0, 0, 0) == 0
+
+
+# ---------------------------------------------------------------- draft
+DRAFT_CASES = [
+    # (t, Hq, Hkv, D, n_sink, window)
+    ([60, 61, 68, 69, 500], 4, 1, 64, 4, 64),     # tiny config's cache, around capacity
+    ([1, 2, 16, 17, 528, 529, 9000], 32, 8, 128, 16, 512),
+    ([1, 5, 6, 7, 100], 8, 8, 128, 1, 4),         # S = 5 < one tile
+    ([3, 300, 5000], 64, 8, 128, 32, 2048),       # G = 8
+    ([10, 20, 4000], 16, 2, 64, 0, 100),          # no sinks
+]
+
+
+@pytest.mark.parametrize("case", DRAFT_CASES, ids=[str(i) for i in range(len(DRAFT_CASES))])
+def test_draft_matches_oracle(spire, case):
+    t, Hq, Hkv, D, ns, w = case
+    di = wl.make_draft(t, Hq, Hkv, D, ns, w, seed=200 + len(t), device=DEV, poison=True)
+    got = parity.gpu_draft(spire, di).cpu().numpy()
+    ref, n_bad = parity.oracle_draft(di)
+    assert n_bad == 0
+    parity.assert_close(got, ref, "draft %s" % (case,))
+
+
+def test_draft_window_covers_context_equals_full_attention(spire):
+    """window >= t: draft == verify at k = 0 over the same keys laid out as pages."""
+    t = [1, 64, 150, 200]
+    ns, w, Hq, Hkv, D = 2, 254, 32, 8, 128
+    di = wl.make_draft(t, Hq, Hkv, D, ns, w, seed=31, device=DEV)
+    dout = parity.gpu_draft(spire, di)
+    S = ns + w
+    pages = (S + 63) // 64
+    B = len(t)
+    kc = torch.zeros((B * pages, Hkv, 64, D), dtype=torch.bfloat16, device=DEV)
+    vc = torch.zeros_like(kc)
+    for b in range(B):
+        for p in range(pages):
+            lo, hi = p * 64, min(S, (p + 1) * 64)
+            kc[b * pages + p, :, :hi - lo] = di.kv[b, 0, :, lo:hi]
+            vc[b * pages + p, :, :hi - lo] = di.kv[b, 1, :, lo:hi]
+    bt = torch.arange(B * pages, dtype=torch.int32, device=DEV).reshape(B, pages)
+    vi = wl.VerifyInputs(q=di.q[:, None].contiguous(), k_cache=kc, v_cache=vc, block_table=bt,
+                         ctx_lens=di.ctx_lens, k=0)
+    vout = parity.gpu_verify(spire, vi)[:, 0]
+    rel, mx = parity.errors(dout.cpu().numpy(), vout.cpu().numpy())
+    assert rel <= 1e-5 and mx <= 1e-5
+
+
+def test_draft_device_error(spire):
+    di = wl.make_draft([0, 40], 8, 2, 128, 4, 64, seed=37, device=DEV)
+    desc = spire.draft_desc(di.q, di.kv)
+    ws = torch.empty(spire.spire_draft_workspace_bytes(desc, 4, 64), dtype=torch.uint8,
+                     device=DEV)
+    out = spire.draft_attention(di.q, di.kv, di.ctx_lens, 4, 64, workspace=ws)
+    assert spire.spire_get_device_error(ws) == 1
+    assert torch.isnan(out[0]).all() and torch.isfinite(out[1]).all()
+
+
+def test_draft_slot_matches_oracle(spire):
+    import oracle
+    for ns, w in [(0, 1), (4, 64), (16, 512), (32, 2048), (16, 4096)]:
+        for p in list(range(0, 3000, 7)) + [10 ** 6 - 1, 262143]:
+            assert spire.spire_draft_slot(p, ns, w) == oracle.draft_slot(p, ns, w)
