@@ -1,6 +1,6 @@
 // spire_abi.cu -- the C ABI of libspire (declared in include/spire.h): host
-// validation, workspace layout, TMA descriptors and the launch sequence
-// plan -> split -> combine on the caller's stream.
+// validation, workspace layout, TMA descriptors and the launch on the
+// caller's stream (a memset of the pair counters, then one attention kernel).
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -11,7 +11,6 @@
 #include <cudaTypedefs.h>
 
 #include "spire.h"
-#include "spire_aux.cuh"
 #include "spire_launch.h"
 
 namespace spire {
@@ -23,19 +22,20 @@ constexpr double kLog2e = 1.4426950408889634;  // log2(e): softmax runs in base 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-    size_t seq_info, items, part_lse, part_o, total;
+    size_t err, cnt, part_lse, part_o, total;
 };
 
-// Work-list bound: with chunk >= ceil(W / kTargetItems), the number of
-// items sum_{b,g} ceil(tiles_b / chunk) is at most kTargetItems + B * Hkv.
+// header (grid size of the last call) | per-CTA error words | per-pair
+// arrival counters | partial slots (two per CTA: a CTA range cuts at most
+// its first and its last pair).
 WsLayout ws_layout(long long B, long long Hkv, long long R, long long D) {
-    const long long max_items = kTargetItems + B * Hkv;
+    const long long slots = 2LL * kMaxCtas;
     WsLayout w{};
     size_t off = kHeaderBytes;
-    w.seq_info = off; off += align256(size_t(B) * 16);
-    w.items = off;    off += align256(size_t(max_items) * 16);
-    w.part_lse = off; off += align256(size_t(max_items * R) * 4);
-    w.part_o = off;   off += align256(size_t(max_items * R * D) * 4);
+    w.err = off;      off += align256(size_t(kMaxCtas) * 4);
+    w.cnt = off;      off += align256(size_t(B * Hkv) * 4);
+    w.part_lse = off; off += align256(size_t(slots * R) * 4);
+    w.part_o = off;   off += align256(size_t(slots * R * D) * 4);
     w.total = off;
     return w;
 }
@@ -85,6 +85,22 @@ bool encode_kv_map(CUtensorMap* map, const void* base, uint64_t D, uint64_t rows
     return r == CUDA_SUCCESS;
 }
 
+// Query rows of pair (b, g): q viewed as {D, Hq, B * kp1}; one box is the
+// G heads of the group for all kp1 block rows, landing as rows r = i*G + hl.
+bool encode_q_map(CUtensorMap* map, const void* q, uint64_t D, uint64_t Hq, uint64_t planes,
+                  uint32_t G, uint32_t kp1) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {D, Hq, planes};
+    cuuint64_t strides[2] = {D * 2, D * 2 * Hq};
+    cuuint32_t box[3] = {64, G, kp1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 struct DeviceInfo {
     int sms = 0;
     int smem_optin = 0;
@@ -128,45 +144,38 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     const int R = rows_per_kv_head(d, kp1);
     const WsLayout w = ws_layout(B, Hkv, R, D);
     char* ws = static_cast<char*>(workspace);
-    int32_t* header = reinterpret_cast<int32_t*>(ws);
-    int4* seq_info = reinterpret_cast<int4*>(ws + w.seq_info);
-    int4* items = reinterpret_cast<int4*>(ws + w.items);
-    float* part_lse = reinterpret_cast<float*>(ws + w.part_lse);
-    float* part_o = reinterpret_cast<float*>(ws + w.part_o);
 
-    PlanParams pp{ctx_lens, seq_info, items, header, B, Hkv, kp1, mode,
-                  mode == kModeVerify ? d->max_pages_per_seq : 0, cap};
-    plan_kernel<<<1, kPlanThreads, 0, stream>>>(pp);
-    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+    AttnParams ap{};
+    ap.q = static_cast<const __nv_bfloat16*>(q);
+    ap.out = out;
+    ap.ctx_lens = ctx_lens;
+    ap.block_table = block_table;
+    ap.header = reinterpret_cast<int32_t*>(ws);
+    ap.err = reinterpret_cast<int32_t*>(ws + w.err);
+    ap.cnt = reinterpret_cast<int32_t*>(ws + w.cnt);
+    ap.part_lse = reinterpret_cast<float*>(ws + w.part_lse);
+    ap.part_o = reinterpret_cast<float*>(ws + w.part_o);
+    ap.B = B;
+    ap.Hq = d->num_q_heads;
+    ap.Hkv = Hkv;
+    ap.G = d->num_q_heads / Hkv;
+    ap.kp1 = kp1;
+    ap.R = R;
+    ap.max_pages = mode == kModeVerify ? d->max_pages_per_seq : 0;
+    ap.num_pages = mode == kModeVerify ? d->num_pages : 0;
+    ap.cap = cap;
+    ap.mode = mode;
+    ap.sl2 = static_cast<float>(static_cast<double>(d->softmax_scale) * kLog2e);
 
-    SplitParams sp{};
-    sp.q = static_cast<const __nv_bfloat16*>(q);
-    sp.out = out;
-    sp.block_table = block_table;
-    sp.seq_info = seq_info;
-    sp.items = items;
-    sp.header = header;
-    sp.part_o = part_o;
-    sp.part_lse = part_lse;
-    sp.B = B;
-    sp.Hq = d->num_q_heads;
-    sp.Hkv = Hkv;
-    sp.G = d->num_q_heads / Hkv;
-    sp.kp1 = kp1;
-    sp.R = R;
-    sp.max_pages = mode == kModeVerify ? d->max_pages_per_seq : 0;
-    sp.num_pages = mode == kModeVerify ? d->num_pages : 0;
-    sp.mode = mode;
-    sp.sl2 = static_cast<float>(static_cast<double>(d->softmax_scale) * kLog2e);
+    CUtensorMap tq;
+    if (!encode_q_map(&tq, q, D, d->num_q_heads, uint64_t(B) * kp1, ap.G, kp1))
+        return SPIRE_ERR_CUDA;
+    if (cudaMemsetAsync(ap.cnt, 0, size_t(B) * Hkv * 4, stream) != cudaSuccess) return SPIRE_ERR_CUDA;
+    const int ctas = di.sms < kMaxCtas ? di.sms : kMaxCtas;
     const int mt = (R + 15) / 16;
-    cudaError_t e = D == 128 ? launch_split_d128(mt, tk, tv, sp, di.sms, stream)
-                             : launch_split_d64(mt, tk, tv, sp, di.sms, stream);
-    if (e != cudaSuccess) return SPIRE_ERR_CUDA;
-
-    CombineParams cp{seq_info, part_o, part_lse, out, B, d->num_q_heads, Hkv, sp.G, kp1, R, D};
-    combine_kernel<<<B * Hkv, 256, 0, stream>>>(cp);
-    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
-    return SPIRE_OK;
+    cudaError_t e = D == 128 ? launch_attn_d128(mt, tk, tv, tq, ap, ctas, stream)
+                             : launch_attn_d64(mt, tk, tv, tq, ap, ctas, stream);
+    return e == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
 }
 
 }  // namespace
@@ -258,10 +267,15 @@ int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {
 spire_status spire_get_device_error(const void* workspace, int32_t* code_out, void* stream) {
     if (!workspace || !code_out) return SPIRE_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    int32_t v = 0;
-    if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    // the header and the per-CTA words are contiguous: one copy
+    int32_t buf[(kHeaderBytes + kMaxCtas * 4) / 4];
+    if (cudaMemcpyAsync(buf, workspace, sizeof(buf), cudaMemcpyDeviceToHost, s) != cudaSuccess)
         return SPIRE_ERR_CUDA;
     if (cudaStreamSynchronize(s) != cudaSuccess) return SPIRE_ERR_CUDA;
+    int n = buf[0];
+    if (n < 0 || n > kMaxCtas) n = kMaxCtas;
+    int32_t v = 0;
+    for (int c = 0; c < n; ++c) v |= buf[kHeaderBytes / 4 + c];
     *code_out = v;
     return SPIRE_OK;
 }

@@ -1,0 +1,278 @@
+// spire_common.cuh -- work decomposition shared by the libspire attention
+// kernels.
+//
+// One speculation round of SPIRe (arXiv 2504.06419) spends its attention time
+// streaming KV caches: the target's full cache once for the k+1 block tokens
+// (Section 2, t_verify) and the draft's bounded sink + window cache once per
+// draft step (Section 3.1).  Both are the same flash-decoding shape: a few
+// query rows per KV head against a run of 64-token K/V tiles.
+//
+// Decomposition.  The unit of work is one 64-token tile of one
+// (sequence b, KV head g) pair.  Pairs are laid end to end in the order
+// (b, g) and their tiles numbered globally 0..W-1.  CTA c of a grid of N
+// takes the contiguous range [floor(cW/N), floor((c+1)W/N)): every SM streams
+// the same number of tiles whatever the spread of lengths.  A pair whose
+// tiles straddle CTA ranges is computed in segments; each segment leaves a
+// normalised partial (O, log-sum-exp) in a slot of the workspace, and the
+// CTA that finishes a pair's last segment (an arrival counter decides)
+// merges them.  The split depends only on ctx_lens, the shapes and N, and
+// partials are merged in slot order, so results are deterministic.
+//
+// Every CTA derives W and its own starting pair from ctx_lens with a
+// block-wide scan; there is no planning kernel.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "spire_ptx.cuh"
+
+namespace spire {
+
+constexpr int kPage = 64;        // tokens per K/V tile (and per page)
+constexpr int kMaxCtas = 512;    // grid cap; the workspace holds 2 partial slots per CTA
+
+constexpr uint32_t kErrCtxLen = 1u;
+constexpr uint32_t kErrPageId = 2u;
+constexpr uint32_t kErrTimeout = 4u;
+
+enum Mode : int32_t { kModeVerify = 0, kModeDraft = 1 };
+
+// Stage flags passed from the producer to the consumers.
+enum : int32_t { kFirst = 1, kLast = 2, kBad = 4, kTerm = 8 };
+
+struct AttnParams {
+    const __nv_bfloat16* q;    // [B, kp1, Hq, D]
+    float* out;                // [B, kp1, Hq, D]
+    const int32_t* ctx_lens;   // [B]
+    const int32_t* block_table;
+    int32_t* header;           // [0]: grid size of the last call
+    int32_t* err;              // [kMaxCtas]: error bits of each CTA of the last call
+    int32_t* cnt;              // [B * Hkv]: segment arrival counters, zero at launch
+    float* part_o;             // [2 * kMaxCtas * R, D]
+    float* part_lse;           // [2 * kMaxCtas * R]
+    int32_t B, Hq, Hkv, G, kp1, R;
+    int32_t max_pages, num_pages;  // verify
+    int32_t cap;                   // draft: cache slots S = n_sink + window
+    int32_t mode;
+    float sl2;                     // softmax_scale * log2(e)
+};
+
+// Tiles of sequence b: ceil(visible length / 64); a sequence whose length
+// breaks the rules occupies one pseudo-tile that yields NaN rows.
+__device__ __forceinline__ int seq_tiles(const AttnParams& p, int L, int* leff, bool* valid) {
+    bool ok;
+    int le;
+    if (p.mode == kModeVerify) {
+        ok = (L >= p.kp1) && ((long long)L <= (long long)p.max_pages * kPage);
+        le = L;
+    } else {
+        ok = L >= 1;
+        le = L < p.cap ? L : p.cap;
+    }
+    *valid = ok;
+    *leff = ok ? le : 0;
+    return ok ? (le + kPage - 1) / kPage : 1;
+}
+
+// CTA whose range holds global tile x (ranges are floor(cW/N) .. floor((c+1)W/N)).
+__device__ __forceinline__ int cta_of(long long x, long long W, int N) {
+    return (int)(((x + 1) * N + W - 1) / W) - 1;
+}
+
+__device__ __forceinline__ long long range_lo(int c, long long W, int N) {
+    return W * c / N;
+}
+
+struct SchedShared {
+    long long W, lo, hi, p0;   // total tiles, this CTA's range, first tile of sequence b0
+    int b0;
+    int N;                     // CTAs with work: min(grid, W), so no range is empty
+    int bad_len;               // some ctx_lens entry breaks the rules
+    long long warp_sums[32];
+};
+
+__device__ __forceinline__ long long block_sum(long long v, SchedShared* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) sh->warp_sums[warp] = v;
+    __syncthreads();
+    long long t = 0;
+    for (int w = 0; w < nw; ++w) t += sh->warp_sums[w];
+    return t;
+}
+
+__device__ __forceinline__ long long block_excl_scan(long long v, SchedShared* sh,
+                                                     long long* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    long long x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    __syncthreads();
+    if (lane == 31) sh->warp_sums[warp] = x;
+    __syncthreads();
+    long long before = 0, t = 0;
+    for (int w = 0; w < nw; ++w) {
+        if (w < warp) before += sh->warp_sums[w];
+        t += sh->warp_sums[w];
+    }
+    *total = t;
+    return before + x - v;
+}
+
+// All threads of the CTA: total work, this CTA's range and the sequence its
+// range starts in.  Leaves the results in *sh (valid after the call).
+__device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
+    long long acc = 0;
+    int bad = 0;
+    for (int b = threadIdx.x; b < p.B; b += blockDim.x) {
+        int le;
+        bool ok;
+        acc += seq_tiles(p, p.ctx_lens[b], &le, &ok);
+        bad |= !ok;
+    }
+    const long long tiles = block_sum(acc, sh);
+    const int any_bad = __syncthreads_or(bad);
+    const long long W = tiles * p.Hkv;
+    const int N = W < (long long)gridDim.x ? (int)W : (int)gridDim.x;
+    const int c = blockIdx.x;
+    const long long lo = c < N ? range_lo(c, W, N) : W, hi = c < N ? range_lo(c + 1, W, N) : W;
+    if (threadIdx.x == 0) {
+        sh->W = W; sh->lo = lo; sh->hi = hi; sh->b0 = 0; sh->p0 = 0; sh->N = N;
+        sh->bad_len = any_bad;
+    }
+    long long carry = 0;
+    for (int base = 0; base < p.B; base += blockDim.x) {
+        const int b = base + threadIdx.x;
+        int le;
+        bool ok;
+        const long long T = b < p.B ? seq_tiles(p, p.ctx_lens[b], &le, &ok) : 0;
+        long long chunk;
+        const long long P = carry + block_excl_scan(T, sh, &chunk);
+        if (b < p.B && lo < hi && P * p.Hkv <= lo && lo < (P + T) * p.Hkv) {
+            sh->b0 = b;
+            sh->p0 = P * p.Hkv;
+        }
+        carry += chunk;
+    }
+    __syncthreads();
+}
+
+// One tile of work as the producer hands it to the consumers.
+struct TileMeta {
+    int b, g, key0, leff;      // sequence, KV head, first key of the tile, visible length
+    int flags, slot, nseg, first_slot;
+};
+
+// Walks this CTA's tile range in order, tracking (b, g, t) incrementally;
+// the segment bookkeeping (divisions) runs once per segment, not per tile.
+struct TileWalker {
+    long long x, hi, lo, W;    // next tile, end of range, start of range, total
+    int N;
+    int b, g, t, T, leff;      // current sequence / KV head / tile-in-pair, tiles per pair
+    bool valid;
+    int slot, nseg, first_slot;
+
+    __device__ void init(const AttnParams& p, const SchedShared& sh) {
+        x = sh.lo; hi = sh.hi; lo = sh.lo; W = sh.W; N = sh.N;
+        b = sh.b0; g = 0; t = 0; T = 1; leff = 0; valid = false;
+        slot = nseg = first_slot = 0;
+        if (x < hi) {
+            T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
+            const long long off = x - sh.p0;
+            g = (int)(off / T);
+            t = (int)(off - (long long)g * T);
+        }
+    }
+    __device__ bool done() const { return x >= hi; }
+
+    // Fills m for tile x and advances; returns the tile index within the pair.
+    __device__ int next(const AttnParams& p, TileMeta* m) {
+        int flags = 0;
+        if (x == lo || t == 0) {
+            flags |= kFirst;
+            // pair_start is the global index of tile 0 of this pair
+            const long long pair_start = x - t, pair_end = pair_start + T;
+            const int c = blockIdx.x;
+            const int c0 = cta_of(pair_start, W, N), c1 = cta_of(pair_end - 1, W, N);
+            slot = (pair_start <= lo) ? 2 * c : 2 * c + 1;   // first segment of this CTA?
+            nseg = c1 - c0 + 1;
+            first_slot = (range_lo(c0, W, N) == pair_start) ? 2 * c0 : 2 * c0 + 1;
+        }
+        if (x == hi - 1 || t == T - 1) flags |= kLast;
+        if (!valid) flags |= kBad;
+        m->b = b; m->g = g; m->key0 = t * kPage; m->leff = leff;
+        m->flags = flags; m->slot = slot; m->nseg = nseg; m->first_slot = first_slot;
+        const int tile = t;
+        ++x;
+        if (++t == T) {
+            t = 0;
+            if (++g == p.Hkv) {
+                g = 0;
+                if (x < hi) {
+                    ++b;
+                    T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
+                }
+            }
+        }
+        return tile;
+    }
+};
+
+// Slot of segment j (0 .. nseg-1) of a pair whose first segment uses first_slot.
+__device__ __forceinline__ int segment_slot(int j, int first_slot) {
+    return j == 0 ? first_slot : 2 * ((first_slot >> 1) + j);
+}
+
+// Output row of query row r (= block row i * G + head-in-group hl) of pair (b, g).
+__device__ __forceinline__ float* out_row(const AttnParams& p, int b, int g, int r, int D) {
+    const int i = r / p.G, hl = r - i * p.G;
+    return p.out + ((long long)(b * p.kp1 + i) * p.Hq + g * p.G + hl) * D;
+}
+
+// Merge the nseg partials of pair (b, g) into the output; executed by
+// `nthreads` threads with ids 0..nthreads-1.  Partials are read around L1.
+template <int D>
+__device__ void merge_pair(const AttnParams& p, int b, int g, int nseg, int first_slot,
+                           int tid, int nthreads) {
+    constexpr int D4 = D / 4;
+    const float NEG_INF = __int_as_float(0xff800000);
+    for (int idx = tid; idx < p.R * D4; idx += nthreads) {
+        const int r = idx / D4, d4 = idx - r * D4;
+        float M = NEG_INF;
+        bool nan = false;
+        for (int j = 0; j < nseg; ++j) {
+            const float l = __ldcg(p.part_lse + (long long)segment_slot(j, first_slot) * p.R + r);
+            nan |= (l != l);
+            M = fmaxf(M, l);
+        }
+        const float Mr = (M == NEG_INF) ? 0.f : M;
+        float den = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int j = 0; j < nseg; ++j) {
+            const long long row = (long long)segment_slot(j, first_slot) * p.R + r;
+            const float w = ex2(__ldcg(p.part_lse + row) - Mr);
+            den += w;
+            const float4 v = __ldcg(reinterpret_cast<const float4*>(p.part_o + row * D) + d4);
+            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+        }
+        float4 res;
+        if (nan || !(den > 0.f)) {
+            const float NANF = __int_as_float(0x7fc00000);
+            res = make_float4(NANF, NANF, NANF, NANF);
+        } else {
+            const float inv = 1.f / den;
+            res = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+        }
+        *reinterpret_cast<float4*>(out_row(p, b, g, r, D) + 4 * d4) = res;
+    }
+}
+
+}  // namespace spire

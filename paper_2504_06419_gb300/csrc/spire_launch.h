@@ -5,34 +5,39 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
-#include "spire_kernels.cuh"
+#include "spire_mma.cuh"
 
 namespace spire {
 
-// Launch the split kernel for head_dim D with MT m-tiles (16 query rows each)
-// on a persistent grid.  Returns the launch error, or cudaErrorInvalidValue
-// for an unsupported MT.
-cudaError_t launch_split_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
-                             const SplitParams& p, int num_sms, cudaStream_t stream);
-cudaError_t launch_split_d128(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
-                              const SplitParams& p, int num_sms, cudaStream_t stream);
+// Launch the attention kernel for head_dim D with MT m-tiles (16 query rows
+// each) on a grid of `ctas` persistent CTAs.  Returns the launch error, or
+// cudaErrorInvalidValue for an unsupported MT.
+cudaError_t launch_attn_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
+                            const CUtensorMap& tq, const AttnParams& p, int ctas,
+                            cudaStream_t stream);
+cudaError_t launch_attn_d128(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
+                             const CUtensorMap& tq, const AttnParams& p, int ctas,
+                             cudaStream_t stream);
 
 // Largest dynamic shared memory one block of this build may use (227 KB).
 constexpr int kMaxDynSmem = 232448;
 
 // Key slices per m-tile: enough consumer warps to keep the tensor pipes and
-// the softmax busy, each warp still owning >= 16 keys of a tile.  The register
+// the softmax busy, each warp still owning >= 16 keys of a tile (measured on
+// GB300: 4 slices for one m-tile, 2 for two or three).  The register
 // file is split across the SM's four sub-partitions, so a block of 9+ warps
 // gets at most 168 registers per thread; from MT = 3 on, one slice per
 // m-tile keeps the block at <= 8 warps.
-constexpr int key_parts(int mt) { return mt <= 2 ? 4 : (mt <= 3 ? 2 : 1); }
+constexpr int key_parts(int mt) { return mt <= 1 ? 4 : (mt <= 3 ? 2 : 1); }
 
 // Deepest stage ring that fits next to the merge scratch.
 template <int D, int MT>
 constexpr int stages() {
     constexpr int kp = key_parts(MT);
     constexpr int nw = MT * kp;
-    constexpr int fixed = nw * 16 * (D + 8) * 4 + nw * 16 * 8 + 8 * 32 + (2 * 8 + 2) * 8 + 1024;
+    constexpr int qbuf = 2 * (D / 64) * MT * 16 * 128;
+    constexpr int fixed = nw * 16 * (D + 8) * 4 + ((nw * 16 * 8 + 1023) / 1024) * 1024 + qbuf +
+                          8 * 32 + 512 + (2 * 8 + 5) * 8 + 1024;
     constexpr int stage = 2 * 64 * D * 2;
     constexpr int n = (kMaxDynSmem - fixed) / stage;
     return n > 8 ? 8 : n;

@@ -1,9 +1,10 @@
-// Split-kernel instantiations for head_dim 64.
+// Attention-kernel instantiations for head_dim 64.
 #include "spire_split_inst.cuh"
 
 namespace spire {
-cudaError_t launch_split_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
-                             const SplitParams& p, int num_sms, cudaStream_t stream) {
-    return launch_split_dispatch<64>(mt, tk, tv, p, num_sms, stream);
+cudaError_t launch_attn_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
+                            const CUtensorMap& tq, const AttnParams& p, int ctas,
+                            cudaStream_t stream) {
+    return launch_attn_dispatch<64>(mt, tk, tv, tq, p, ctas, stream);
 }
 }  // namespace spire

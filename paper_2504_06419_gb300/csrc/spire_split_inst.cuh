@@ -1,4 +1,4 @@
-// spire_split_inst.cuh -- instantiates and launches the split kernel for one
+// spire_split_inst.cuh -- instantiates and launches the attention kernel for one
 // head_dim; included by spire_split_d64.cu / spire_split_d128.cu.
 #pragma once
 
@@ -9,14 +9,14 @@
 namespace spire {
 
 template <int D, int MT>
-cudaError_t launch_split_t(const CUtensorMap& tk, const CUtensorMap& tv, const SplitParams& p,
-                           int num_sms, cudaStream_t stream) {
+cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
+                          const AttnParams& p, int ctas, cudaStream_t stream) {
     constexpr int KP = key_parts(MT);
     constexpr int NST = stages<D, MT>();
     static_assert(NST >= 2, "stage ring does not fit in shared memory");
-    using C = SplitCfg<D, MT, KP, NST>;
+    using C = MmaCfg<D, MT, KP, NST>;
     static_assert(C::SMEM <= kMaxDynSmem, "shared memory budget exceeded");
-    auto kern = split_kernel<D, MT, KP, NST>;
+    auto kern = attn_mma_kernel<D, MT, KP, NST>;
     // the shared-memory opt-in is per device; remember it for the first 64
     static std::atomic<unsigned long long> done{0ull};
     int dev = 0;
@@ -29,22 +29,23 @@ cudaError_t launch_split_t(const CUtensorMap& tk, const CUtensorMap& tv, const S
         done.fetch_or(bit, std::memory_order_acq_rel);
     }
     // one CTA per SM: the stage ring takes most of the shared memory
-    kern<<<num_sms, C::THREADS, C::SMEM, stream>>>(tk, tv, p);
+    kern<<<ctas, C::THREADS, C::SMEM, stream>>>(tk, tv, tq, p);
     return cudaGetLastError();
 }
 
 template <int D>
-cudaError_t launch_split_dispatch(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
-                                  const SplitParams& p, int num_sms, cudaStream_t stream) {
+cudaError_t launch_attn_dispatch(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
+                                 const CUtensorMap& tq, const AttnParams& p, int ctas,
+                                 cudaStream_t stream) {
     switch (mt) {
-        case 1: return launch_split_t<D, 1>(tk, tv, p, num_sms, stream);
-        case 2: return launch_split_t<D, 2>(tk, tv, p, num_sms, stream);
-        case 3: return launch_split_t<D, 3>(tk, tv, p, num_sms, stream);
-        case 4: return launch_split_t<D, 4>(tk, tv, p, num_sms, stream);
-        case 5: return launch_split_t<D, 5>(tk, tv, p, num_sms, stream);
-        case 6: return launch_split_t<D, 6>(tk, tv, p, num_sms, stream);
-        case 7: return launch_split_t<D, 7>(tk, tv, p, num_sms, stream);
-        case 8: return launch_split_t<D, 8>(tk, tv, p, num_sms, stream);
+        case 1: return launch_attn_t<D, 1>(tk, tv, tq, p, ctas, stream);
+        case 2: return launch_attn_t<D, 2>(tk, tv, tq, p, ctas, stream);
+        case 3: return launch_attn_t<D, 3>(tk, tv, tq, p, ctas, stream);
+        case 4: return launch_attn_t<D, 4>(tk, tv, tq, p, ctas, stream);
+        case 5: return launch_attn_t<D, 5>(tk, tv, tq, p, ctas, stream);
+        case 6: return launch_attn_t<D, 6>(tk, tv, tq, p, ctas, stream);
+        case 7: return launch_attn_t<D, 7>(tk, tv, tq, p, ctas, stream);
+        case 8: return launch_attn_t<D, 8>(tk, tv, tq, p, ctas, stream);
         default: return cudaErrorInvalidValue;
     }
 }
