@@ -173,8 +173,18 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     if (cudaMemsetAsync(ap.cnt, 0, size_t(B) * Hkv * 4, stream) != cudaSuccess) return SPIRE_ERR_CUDA;
     const int ctas = di.sms < kMaxCtas ? di.sms : kMaxCtas;
     const int mt = (R + 15) / 16;
-    cudaError_t e = D == 128 ? launch_attn_d128(mt, tk, tv, tq, ap, ctas, stream)
-                             : launch_attn_d64(mt, tk, tv, tq, ap, ctas, stream);
+    // tcgen05 path when a KV head serves enough query rows to make QK^T and PV
+    // real contractions; the warp-MMA path for the few-row draft step, whose
+    // short pairs favour its lighter per-pair epilogue (measured on GB300)
+    const bool use_tc = R > 8;
+    cudaError_t e;
+    const int nc = R <= 32 ? 4 : (R <= 64 ? 2 : 1);   // query copies of the tcgen05 kernel
+    if (use_tc)
+        e = D == 128 ? launch_attn_tc_d128(nc, tk, tv, tq, ap, ctas, stream)
+                     : launch_attn_tc_d64(nc, tk, tv, tq, ap, ctas, stream);
+    else
+        e = D == 128 ? launch_attn_d128(mt, tk, tv, tq, ap, ctas, stream)
+                     : launch_attn_d64(mt, tk, tv, tq, ap, ctas, stream);
     return e == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
 }
 

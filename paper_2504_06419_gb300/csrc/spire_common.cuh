@@ -226,6 +226,113 @@ struct TileWalker {
     }
 };
 
+// Shared-memory layout the producer fills: NST stages of [K tile | V tile]
+// (each D/64 boxes of 64 keys x 128 bytes, 128-byte swizzled) and two Q
+// buffers of D/64 halves, each half QHALF bytes of 128-byte rows holding
+// `qcopies` copies of the pair's R query rows, `qcopy_rows` rows apart.
+struct ProducerSmem {
+    uint32_t stages;       // shared address of stage 0
+    uint32_t q;            // shared address of Q buffer 0
+    uint32_t qhalf;        // bytes per 64-column half of a Q buffer
+    int4* meta;            // 2 int4 per stage
+    uint32_t bar_full, bar_empty, bar_qfull, bar_qempty;
+    int qcopies;           // copies of the query rows per Q buffer
+    int qcopy_rows;        // rows between consecutive copies
+};
+
+// Meta word layout: meta[2s] = {b, g, key0, leff}; meta[2s+1] = {flags |
+// (qflag << 8), slot, nseg, first_slot} where qflag = 16 | Q buffer when the
+// tile starts a segment whose query rows were loaded.
+//
+// Streams this CTA's tiles; run by one thread.  Returns the error bits it
+// found.  The stage ring protocol: wait `empty` (parity ph ^ 1), fill, arrive
+// on `full` with the byte count; a tile that must not be read (bad length or
+// page) arrives without a copy and carries kBad.  The run ends with a stage
+// that carries kTerm.
+template <int D, int NST>
+__device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CUtensorMap* tmap_k,
+                            const CUtensorMap* tmap_v, const CUtensorMap* tmap_q,
+                            const ProducerSmem& sm) {
+    constexpr uint32_t TILE = kPage * D * 2, STAGE = 2 * TILE;
+    uint32_t err = sh.bad_len ? kErrCtxLen : 0u;
+    prefetch_tensormap(tmap_k);
+    prefetch_tensormap(tmap_v);
+    prefetch_tensormap(tmap_q);
+    const uint64_t pol = policy_evict_first();
+    const uint32_t qbytes = (D / 64) * sm.qcopies * p.R * 128;
+    const uint32_t qbuf = (D / 64) * sm.qhalf;
+    uint32_t st = 0, ph = 0, qs = 0, qph = 0;      // stage ring / Q double buffer
+    uint32_t armed = 0, armed_parity = 0;          // stages with a TMA load issued, and its phase
+    uint32_t qarmed = 0, qarmed_parity = 0;
+    bool ok = true;
+    TileWalker wk;
+    wk.init(p, sh);
+    while (!wk.done()) {
+        if (!mbar_wait(sm.bar_empty + 8 * st, ph ^ 1)) { ok = false; break; }
+        TileMeta m;
+        const int t = wk.next(p, &m);
+        int qflag = 0;
+        if ((m.flags & kFirst) && !(m.flags & kBad)) {
+            // the pair's query rows r = i*G + hl, one box per 64 columns
+            if (!mbar_wait(sm.bar_qempty + 8 * qs, qph ^ 1)) { ok = false; break; }
+            mbar_arrive_expect_tx(sm.bar_qfull + 8 * qs, qbytes);
+            for (int c = 0; c < sm.qcopies; ++c)
+#pragma unroll
+                for (int h = 0; h < D / 64; ++h)
+                    tma_load_3d(sm.q + qs * qbuf + h * sm.qhalf + c * sm.qcopy_rows * 128, tmap_q,
+                                h * 64, m.g * p.G, m.b * p.kp1, sm.bar_qfull + 8 * qs, pol);
+            qarmed |= 1u << qs;
+            qarmed_parity = (qarmed_parity & ~(1u << qs)) | (qph << qs);
+            qflag = 16 | qs;
+            if (++qs == 2) { qs = 0; qph ^= 1; }
+        }
+        int zk = 0, zv = 0, y = 0;
+        if (!(m.flags & kBad)) {
+            if (p.mode == kModeVerify) {
+                const int page = p.block_table[(long long)m.b * p.max_pages + t];
+                if (page < 0 || page >= p.num_pages) {
+                    m.flags |= kBad;
+                    err |= kErrPageId;
+                }
+                zk = zv = page * p.Hkv + m.g;
+            } else {
+                y = m.key0;
+                zk = (m.b * 2 + 0) * p.Hkv + m.g;
+                zv = (m.b * 2 + 1) * p.Hkv + m.g;
+            }
+        }
+        sm.meta[2 * st] = make_int4(m.b, m.g, m.key0, m.leff);
+        sm.meta[2 * st + 1] = make_int4(m.flags | (qflag << 8), m.slot, m.nseg, m.first_slot);
+        if (m.flags & kBad) {
+            mbar_arrive(sm.bar_full + 8 * st);
+        } else {
+            const uint32_t dk = sm.stages + st * STAGE, dv = dk + TILE;
+            mbar_arrive_expect_tx(sm.bar_full + 8 * st, STAGE);
+#pragma unroll
+            for (int h = 0; h < D / 64; ++h) {
+                tma_load_3d(dk + h * 8192, tmap_k, h * 64, y, zk, sm.bar_full + 8 * st, pol);
+                tma_load_3d(dv + h * 8192, tmap_v, h * 64, y, zv, sm.bar_full + 8 * st, pol);
+            }
+            armed |= 1u << st;
+            armed_parity = (armed_parity & ~(1u << st)) | (ph << st);
+        }
+        if (++st == NST) { st = 0; ph ^= 1; }
+    }
+    if (ok && mbar_wait(sm.bar_empty + 8 * st, ph ^ 1)) {
+        sm.meta[2 * st + 1] = make_int4(kTerm, 0, 0, 0);
+        mbar_arrive(sm.bar_full + 8 * st);
+    } else {
+        // Consumers stopped answering: record it and wait (bounded) for our
+        // own copies to land before the CTA's shared memory goes away.
+        err |= kErrTimeout;
+        for (int s = 0; s < NST; ++s)
+            if (armed & (1u << s)) mbar_wait(sm.bar_full + 8 * s, (armed_parity >> s) & 1u);
+        for (int s = 0; s < 2; ++s)
+            if (qarmed & (1u << s)) mbar_wait(sm.bar_qfull + 8 * s, (qarmed_parity >> s) & 1u);
+    }
+    return err;
+}
+
 // Slot of segment j (0 .. nseg-1) of a pair whose first segment uses first_slot.
 __device__ __forceinline__ int segment_slot(int j, int first_slot) {
     return j == 0 ? first_slot : 2 * ((first_slot >> 1) + j);

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include "spire_mma.cuh"
+#include "spire_tc.cuh"
 
 namespace spire {
 
@@ -18,6 +19,15 @@ cudaError_t launch_attn_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv
 cudaError_t launch_attn_d128(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
                              const CUtensorMap& tq, const AttnParams& p, int ctas,
                              cudaStream_t stream);
+
+// tcgen05 kernel (any R <= 128): one CTA per SM; nc = copies of the query
+// rows (4 for R <= 32, 2 for R <= 64, else 1).
+cudaError_t launch_attn_tc_d64(int nc, const CUtensorMap& tk, const CUtensorMap& tv,
+                               const CUtensorMap& tq, const AttnParams& p, int ctas,
+                               cudaStream_t stream);
+cudaError_t launch_attn_tc_d128(int nc, const CUtensorMap& tk, const CUtensorMap& tv,
+                                const CUtensorMap& tq, const AttnParams& p, int ctas,
+                                cudaStream_t stream);
 
 // Largest dynamic shared memory one block of this build may use (227 KB).
 constexpr int kMaxDynSmem = 232448;
@@ -41,6 +51,17 @@ constexpr int stages() {
     constexpr int stage = 2 * 64 * D * 2;
     constexpr int n = (kMaxDynSmem - fixed) / stage;
     return n > 8 ? 8 : n;
+}
+
+// Deepest stage ring of the tcgen05 kernel next to its two Q buffers and the
+// copy-merge scratch.
+template <int D, int NC>
+constexpr int tc_stages() {
+    constexpr int scr = 2 * (NC - 1) * 32 * (4 / NC) * 33 * 4;
+    constexpr int fixed = 2 * (D / 64) * 16384 + scr + 128 * 8 + 8 * 32 + 512 + 16 +
+                          (3 * 8 + 19) * 8 + 1024;
+    constexpr int n = (kMaxDynSmem - fixed) / (2 * 64 * D * 2);
+    return n > 6 ? 6 : n;
 }
 
 }  // namespace spire

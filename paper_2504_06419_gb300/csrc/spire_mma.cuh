@@ -96,75 +96,9 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     if (warp == C::NW) {
         // ------------------------------------------------------ producer
         if (lane != 0) return;
-        uint32_t err = sh->bad_len ? kErrCtxLen : 0u;
-        prefetch_tensormap(&tmap_k);
-        prefetch_tensormap(&tmap_v);
-        prefetch_tensormap(&tmap_q);
-        const uint64_t pol = policy_evict_first();
-        const uint32_t qbytes = (D / 64) * p.R * 128;
-        uint32_t st = 0, ph = 0, qs = 0, qph = 0;     // stage ring / Q double buffer
-        uint32_t armed = 0, armed_parity = 0;   // stages with a TMA load issued, and its phase
-        bool ok = true;
-        TileWalker wk;
-        wk.init(p, *sh);
-        while (!wk.done()) {
-            if (!mbar_wait(bar_empty + 8 * st, ph ^ 1)) { ok = false; break; }
-            TileMeta m;
-            const int t = wk.next(p, &m);
-            int qflag = 0;
-            if ((m.flags & kFirst) && !(m.flags & kBad)) {
-                // the pair's query rows r = i*G + hl, one box per 64 columns
-                if (!mbar_wait(bar_qempty + 8 * qs, qph ^ 1)) { ok = false; break; }
-                mbar_arrive_expect_tx(bar_qfull + 8 * qs, qbytes);
-#pragma unroll
-                for (int h = 0; h < D / 64; ++h)
-                    tma_load_3d(qsm + qs * C::QBUF + h * C::QHALF, &tmap_q, h * 64, m.g * p.G,
-                                m.b * p.kp1, bar_qfull + 8 * qs, pol);
-                qflag = 16 | qs;
-                if (++qs == 2) { qs = 0; qph ^= 1; }
-            }
-            int zk = 0, zv = 0, y = 0;
-            if (!(m.flags & kBad)) {
-                if (p.mode == kModeVerify) {
-                    const int page = p.block_table[(long long)m.b * p.max_pages + t];
-                    if (page < 0 || page >= p.num_pages) {
-                        m.flags |= kBad;
-                        err |= kErrPageId;
-                    }
-                    zk = zv = page * p.Hkv + m.g;
-                } else {
-                    y = m.key0;
-                    zk = (m.b * 2 + 0) * p.Hkv + m.g;
-                    zv = (m.b * 2 + 1) * p.Hkv + m.g;
-                }
-            }
-            meta[2 * st] = make_int4(m.b, m.g, m.key0, m.leff);
-            meta[2 * st + 1] = make_int4(m.flags | (qflag << 8), m.slot, m.nseg, m.first_slot);
-            if (m.flags & kBad) {
-                mbar_arrive(bar_full + 8 * st);
-            } else {
-                const uint32_t dk = base + st * C::STAGE, dv = dk + C::TILE;
-                mbar_arrive_expect_tx(bar_full + 8 * st, C::STAGE);
-#pragma unroll
-                for (int h = 0; h < D / 64; ++h) {
-                    tma_load_3d(dk + h * 8192, &tmap_k, h * 64, y, zk, bar_full + 8 * st, pol);
-                    tma_load_3d(dv + h * 8192, &tmap_v, h * 64, y, zv, bar_full + 8 * st, pol);
-                }
-                armed |= 1u << st;
-                armed_parity = (armed_parity & ~(1u << st)) | (ph << st);
-            }
-            if (++st == NST) { st = 0; ph ^= 1; }
-        }
-        if (ok && mbar_wait(bar_empty + 8 * st, ph ^ 1)) {
-            meta[2 * st + 1] = make_int4(kTerm, 0, 0, 0);
-            mbar_arrive(bar_full + 8 * st);
-        } else {
-            // Consumers stopped answering: record it and wait (bounded) for
-            // our own copies to land before the CTA's shared memory goes away.
-            err |= kErrTimeout;
-            for (int s = 0; s < NST; ++s)
-                if (armed & (1u << s)) mbar_wait(bar_full + 8 * s, (armed_parity >> s) & 1u);
-        }
+        const ProducerSmem psm{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
+                               bar_empty, bar_qfull, bar_qempty, 1, 0};
+        const uint32_t err = produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, psm);
         if (err) atomicOr(&p.err[blockIdx.x], (int)err);
         return;
     }

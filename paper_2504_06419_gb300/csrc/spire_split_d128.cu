@@ -7,4 +7,9 @@ cudaError_t launch_attn_d128(int mt, const CUtensorMap& tk, const CUtensorMap& t
                             cudaStream_t stream) {
     return launch_attn_dispatch<128>(mt, tk, tv, tq, p, ctas, stream);
 }
+cudaError_t launch_attn_tc_d128(int nc, const CUtensorMap& tk, const CUtensorMap& tv,
+                               const CUtensorMap& tq, const AttnParams& p, int ctas,
+                               cudaStream_t stream) {
+    return launch_tc_dispatch<128>(nc, tk, tv, tq, p, ctas, stream);
+}
 }  // namespace spire

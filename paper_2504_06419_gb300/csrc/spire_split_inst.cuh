@@ -33,6 +33,40 @@ cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CU
     return cudaGetLastError();
 }
 
+template <int D, int NC>
+cudaError_t launch_tc_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
+                        const AttnParams& p, int ctas, cudaStream_t stream) {
+    constexpr int NST = tc_stages<D, NC>();
+    static_assert(NST >= 2, "stage ring does not fit in shared memory");
+    using C = TcCfg<D, NC, NST>;
+    static_assert(C::SMEM <= kMaxDynSmem, "shared memory budget exceeded");
+    auto kern = attn_tc_kernel<D, NC, NST>;
+    static std::atomic<unsigned long long> done{0ull};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = dev < 64 ? (1ull << dev) : 0ull;
+    if (!bit || !(done.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (e != cudaSuccess) return e;
+        done.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    kern<<<ctas, C::THREADS, C::SMEM, stream>>>(tk, tv, tq, p);
+    return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_tc_dispatch(int nc, const CUtensorMap& tk, const CUtensorMap& tv,
+                               const CUtensorMap& tq, const AttnParams& p, int ctas,
+                               cudaStream_t stream) {
+    switch (nc) {
+        case 4: return launch_tc_t<D, 4>(tk, tv, tq, p, ctas, stream);
+        case 2: return launch_tc_t<D, 2>(tk, tv, tq, p, ctas, stream);
+        case 1: return launch_tc_t<D, 1>(tk, tv, tq, p, ctas, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
 template <int D>
 cudaError_t launch_attn_dispatch(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
                                  const CUtensorMap& tq, const AttnParams& p, int ctas,

@@ -1,0 +1,530 @@
+// spire_tc.cuh -- attention kernel on the Blackwell tensor cores (tcgen05,
+// accumulators and P in tensor memory).
+//
+// Roles in a CTA (one CTA per SM, 7 warps):
+//   warp 0 (producer)   the TMA producer shared with the warp-MMA kernel:
+//                       K/V tiles into an NST-deep stage ring and each pair's
+//                       query rows into one of two Q buffers.
+//   warp 1 (QK issuer)  allocates tensor memory; one thread issues
+//                         S[sb]  = Q K^T   (M=128 rows, N=64 keys, K=D)
+//   warp 6 (PV issuer)  one thread issues
+//                         O     += P V     (M=128, N=D, K=64)
+//                       Both use tcgen05.mma with the A operand (Q, P) in
+//                       tensor memory and B (K, V tiles) in shared memory and
+//                       signal completion with tcgen05.commit.  One thread can
+//                       issue an MMA only every ~45 cycles, so QK and PV get a
+//                       thread each; they follow the stage ring independently
+//                       and the softmax of tile n overlaps QK of tile n+1.
+//   warps 2..5          softmax, one thread per tensor-memory lane.
+//
+// Query copies.  A pair has R = G*(k+1) <= 128 query rows, but the tile has
+// 128.  The spare rows are used: the Q buffer holds NC = 128 / (32*ceil(R/32))
+// copies of the R rows (NC = 4 for R <= 32, 2 for R <= 64, else 1), and copy c
+// is responsible only for keys [c*64/NC, (c+1)*64/NC) of every tile -- its P
+// is zero elsewhere.  So each of the four softmax warps handles 64/NC keys per
+// tile instead of one warp handling all 64.  Every copy keeps its own running
+// max m and sum l (fp32, base 2); at the end of a segment the copies are
+// merged through shared memory with weights 2^(m_c - max_c m_c).
+//
+// Per tile, a softmax thread reads its slice of the S row from tensor memory,
+// masks keys past its row's causal / length limit, updates m lazily (only
+// when a score exceeds m by more than 2^8, so O is rescaled in tensor memory
+// only rarely and P stays <= 2^8), and writes P = P_hi + P_lo (two bf16 parts,
+// ~16 mantissa bits together) back to tensor memory.
+//
+// Tensor memory: S double buffer in columns [0, 128), O in [128, 128 + D),
+// P double buffer in [256, 384) (per buffer: 32 columns of packed P_hi, then
+// 32 of P_lo; key 2j in the low half of column j), Q double buffer in
+// [384, 384 + D) (D/2 packed columns per buffer).  The softmax warps copy each
+// pair's query rows from the TMA buffer in shared memory into tensor memory
+// once per segment, so QK reads only the K tile from shared memory.  Double buffers let the
+// softmax of tile n+1 run while PV of tile n still reads its P.  Every tile,
+// bad or not, is acknowledged on its stage's p_full barrier by the softmax
+// warps and the QK issuer before the PV issuer releases the stage.
+#pragma once
+
+#include "spire_common.cuh"
+
+namespace spire {
+
+template <int D, int NC, int NST>
+struct TcCfg {
+    static constexpr int THREADS = 224;
+    static constexpr int TILE = kPage * D * 2;     // one K (or V) tile
+    static constexpr int STAGE = 2 * TILE;
+    static constexpr int QHALF = 128 * 128;        // 128 rows x 64 columns of bf16
+    static constexpr int QBUF = (D / 64) * QHALF;
+    static constexpr int KW = kPage / NC;          // keys of a tile per copy
+    static constexpr int RB = 4 / NC;              // 32-row blocks per copy
+    static constexpr int SCR_ROWS = (NC - 1) * 32 * RB;   // rows of copies 1 .. NC-1
+    static constexpr int SCR_LD = 33;              // floats per scratch row (32 + pad)
+    static constexpr int OFF_Q = NST * STAGE;
+    static constexpr int OFF_SCR = OFF_Q + 2 * QBUF;
+    static constexpr int OFF_ML = OFF_SCR + 2 * SCR_ROWS * SCR_LD * 4;
+    static constexpr int OFF_META = OFF_ML + 128 * 8;
+    static constexpr int OFF_SCHED = OFF_META + NST * 32;
+    static constexpr int OFF_MISC = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16;
+    static constexpr int OFF_BAR = OFF_MISC + 16;
+    static constexpr int NBAR = 3 * NST + 19;
+    static constexpr int SMEM = OFF_BAR + NBAR * 8 + 1024;   // + alignment slack
+    static constexpr uint32_t TMEM_COLS = 512;
+    static constexpr int S_COL = 0, O_COL = 128, P_COL = 256, Q_COL = 384;
+    static_assert(NC == 1 || NC == 2 || NC == 4, "1, 2 or 4 query copies");
+    static_assert(STAGE % 1024 == 0 && OFF_Q % 1024 == 0,
+                  "swizzled regions must be 1024-byte aligned");
+    static_assert(O_COL + D <= P_COL && Q_COL + D <= (int)TMEM_COLS, "tensor memory budget");
+};
+
+constexpr float kLazy = 8.0f;   // log2 units: rescale O only when the max grows by > 2^8
+
+template <int D, int NC, int NST>
+__global__ void __launch_bounds__(224, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                   const __grid_constant__ CUtensorMap tmap_v,
+                   const __grid_constant__ CUtensorMap tmap_q, const AttnParams p) {
+    using C = TcCfg<D, NC, NST>;
+    constexpr int KW = C::KW;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* const sbase = smem_raw + (base - raw);
+    int4* const meta = reinterpret_cast<int4*>(sbase + C::OFF_META);
+    SchedShared* const sh = reinterpret_cast<SchedShared*>(sbase + C::OFF_SCHED);
+    uint32_t* const misc = reinterpret_cast<uint32_t*>(sbase + C::OFF_MISC);  // [0] TMEM base, [1] merge flag
+    float* const scr = reinterpret_cast<float*>(sbase + C::OFF_SCR);
+    float2* const mls = reinterpret_cast<float2*>(sbase + C::OFF_ML);
+    const uint32_t qsm = base + C::OFF_Q;
+    const uint32_t bar0 = base + C::OFF_BAR;
+    const uint32_t bar_full = bar0, bar_empty = bar0 + 8 * NST, bar_pfull = bar0 + 16 * NST;
+    const uint32_t bar_qfull = bar0 + 24 * NST, bar_qempty = bar_qfull + 16;
+    const uint32_t bar_sfull = bar_qempty + 16, bar_sfree = bar_sfull + 16;
+    const uint32_t bar_obar = bar_sfree + 16;
+    const uint32_t bar_grp = bar_obar + 16, bar_drain = bar_grp + 8;
+    const uint32_t bar_qtfull = bar_drain + 16, bar_qtfree = bar_qtfull + 16;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NST; ++s) {
+            mbar_init(bar_full + 8 * s, 1);
+            mbar_init(bar_empty + 8 * s, 1);
+            mbar_init(bar_pfull + 8 * s, 5);   // softmax warps and the QK issuer are done with it
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(bar_qfull + 8 * b, 1);
+            mbar_init(bar_qempty + 8 * b, 4);    // softmax warps copied the rows out
+            mbar_init(bar_qtfull + 8 * b, 4);    // rows are in tensor-memory Q buffer b
+            mbar_init(bar_qtfree + 8 * b, 1);    // the last QK reading it has completed
+            mbar_init(bar_sfull + 8 * b, 1);
+            mbar_init(bar_sfree + 8 * b, 4);
+            mbar_init(bar_obar + 8 * b, 1);    // PV reading P buffer b has completed
+        }
+        mbar_init(bar_grp, 128);
+        mbar_init(bar_drain, 1);
+        mbar_init(bar_drain + 8, 1);
+        fence_barrier_init();
+        if (blockIdx.x == 0) p.header[0] = gridDim.x;
+        p.err[blockIdx.x] = 0;
+    }
+    // Q rows of padding stay zero for the whole kernel
+    for (int i = threadIdx.x; i < (2 * C::QBUF) / 16; i += blockDim.x)
+        reinterpret_cast<uint4*>(sbase + C::OFF_Q)[i] = make_uint4(0u, 0u, 0u, 0u);
+    fence_proxy_async();
+    if (warp == 1) {
+        tmem_alloc(base + C::OFF_MISC, C::TMEM_COLS);
+        tmem_relinquish();
+        tc_fence_before();
+    }
+    sched_setup(p, sh);   // ends with __syncthreads()
+    tc_fence_after();
+    const uint32_t tmem = misc[0];
+    uint32_t err = 0;
+
+    if (warp == 0) {
+        // ------------------------------------------------------ producer
+        if (lane == 0) {
+            const ProducerSmem ps{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
+                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC};
+            err |= produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------ QK issuer
+        if (lane == 0) {
+            constexpr uint32_t ID_QK = idesc_bf16(128, 64, false);
+            uint32_t st = 0, ph = 0, cq0 = 0, cq1 = 0, n_qk = 0;
+            int qb = 0;
+            bool have_q = false, ok = true;
+            for (;;) {
+                if (!mbar_wait(bar_full + 8 * st, ph)) { ok = false; break; }
+                const int4 mb = meta[2 * st + 1];
+                const int flags = mb.x & 0xff, qflag = mb.x >> 8;
+                if (flags & kTerm) break;
+                if (flags & kFirst) {
+                    have_q = qflag & 16;
+                    if (have_q) {
+                        qb = qflag & 1;
+                        const uint32_t par = qb ? cq1 : cq0;
+                        if (!mbar_wait(bar_qtfull + 8 * qb, par)) { ok = false; break; }
+                        if (qb) cq1 ^= 1; else cq0 ^= 1;
+                    }
+                }
+                if (!(flags & kBad)) {
+                    const uint32_t sb = n_qk & 1;
+                    if (!mbar_wait(bar_sfree + 8 * sb, ((n_qk >> 1) & 1) ^ 1)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t kaddr = base + st * C::STAGE;
+                    const uint32_t qcol = tmem + C::Q_COL + qb * (D / 2);
+#pragma unroll
+                    for (int ks = 0; ks < D / 16; ++ks) {
+                        const uint64_t b = sdesc_sw128(kaddr + (ks >> 2) * 8192 + (ks & 3) * 32, 16, 1024);
+                        umma_bf16_ts(tmem + C::S_COL + sb * 64, qcol + ks * 8, b, ID_QK, ks > 0);
+                    }
+                    umma_commit(bar_sfull + 8 * sb);
+                    ++n_qk;
+                }
+                if ((flags & kLast) && have_q) umma_commit(bar_qtfree + 8 * qb);
+                mbar_arrive(bar_pfull + 8 * st);   // done with this stage's meta and K tile
+                if (++st == NST) { st = 0; ph ^= 1; }
+            }
+            if (!ok) err |= kErrTimeout;
+            // every issued tensor-core operation has finished before TMEM is freed
+            umma_commit(bar_drain);
+            if (!mbar_wait(bar_drain, 0)) err |= kErrTimeout;
+        }
+        __syncwarp();
+    } else if (warp == 6) {
+        // ------------------------------------------------------ PV issuer
+        if (lane == 0) {
+            constexpr uint32_t ID_PV = idesc_bf16(128, D, true);
+            uint32_t st = 0, ph = 0, n_pv = 0;
+            int seg_nonbad = 0;
+            bool ok = true;
+            for (;;) {
+                if (!mbar_wait(bar_full + 8 * st, ph)) { ok = false; break; }
+                const int flags = meta[2 * st + 1].x & 0xff;
+                if (flags & kTerm) break;
+                if (flags & kFirst) seg_nonbad = 0;
+                // P written (or the tile acknowledged) by all its readers
+                if (!mbar_wait(bar_pfull + 8 * st, ph)) { ok = false; break; }
+                tc_fence_after();
+                if (!(flags & kBad)) {
+                    const uint32_t accum = seg_nonbad > 0;   // first PV of a segment overwrites O
+                    ++seg_nonbad;
+                    const uint32_t vaddr = base + st * C::STAGE + C::TILE;
+                    const uint32_t pcol = tmem + C::P_COL + (n_pv & 1) * 64;
+#pragma unroll
+                    for (int part = 0; part < 2; ++part) {        // P_hi, then P_lo
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t b = sdesc_sw128(vaddr + kk * 2048, 8192, 1024);
+                            umma_bf16_ts(tmem + C::O_COL, pcol + part * 32 + kk * 8, b, ID_PV,
+                                         (accum | part | kk) != 0);
+                        }
+                    }
+                    umma_commit(bar_obar + 8 * (n_pv & 1));
+                    umma_commit(bar_empty + 8 * st);
+                    ++n_pv;
+                } else {
+                    mbar_arrive(bar_empty + 8 * st);
+                }
+                if (++st == NST) { st = 0; ph ^= 1; }
+            }
+            if (!ok) err |= kErrTimeout;
+            umma_commit(bar_drain + 8);
+            if (!mbar_wait(bar_drain + 8, 0)) err |= kErrTimeout;
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------ softmax warps
+        const int quarter = warp & 3;                 // TMEM lanes 32*quarter .. +31
+        const int tl = 32 * quarter + lane;           // this thread's TMEM lane
+        const int copy = quarter / C::RB;             // query copy (key slice) of the lane
+        const int r = 32 * (quarter % C::RB) + lane;  // query row within the copy
+        const bool active = 32 * (quarter % C::RB) < p.R;   // warp holds a real row
+        const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16);
+        const int gtid = threadIdx.x - 64;            // 0..127
+        const float NEG_INF = __int_as_float(0xff800000);
+        const float NANF = __int_as_float(0x7fc00000);
+        const float sl2 = p.sl2;
+        const int i_r = min(r / p.G, p.kp1 - 1);      // block row of query row r
+        const int kofs = copy * KW;                   // first key of this copy's slice
+        uint32_t st = 0, ph = 0, n_qk = 0, n_pv = 0, gph = 0;
+        uint32_t qu0 = 0, qu1 = 0;                    // fills of Q buffer 0 / 1 so far
+        float m = NEG_INF, l = 0.f;
+        bool poison = false;
+        int seg_pv = 0;
+        int cur_b = 0, cur_g = 0, cur_slot = 0, cur_nseg = 1, cur_first = 0, leff = 0, lim = 0;
+        bool ok = true;
+        auto grp_sync = [&]() -> bool {
+            mbar_arrive(bar_grp);
+            const bool rr = mbar_wait(bar_grp, gph & 1);
+            ++gph;
+            return rr;
+        };
+        // P columns outside this copy's key slice stay zero
+        {
+            uint32_t z[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) z[j] = 0u;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_st32u(trow + C::P_COL + 32 * c, z);
+            tmem_wait_st();
+        }
+        for (;;) {
+            if (!mbar_wait(bar_full + 8 * st, ph)) { ok = false; break; }
+            const int4 ma = meta[2 * st], mb = meta[2 * st + 1];
+            const int flags = mb.x & 0xff;
+            if (flags & kTerm) break;
+            if (flags & kFirst) {
+                cur_b = ma.x; cur_g = ma.y; leff = ma.w;
+                cur_slot = mb.y; cur_nseg = mb.z; cur_first = mb.w;
+                m = NEG_INF; l = 0.f; poison = false; seg_pv = 0;
+                lim = leff - (p.kp1 - 1) + i_r;
+                const int qflag = mb.x >> 8;
+                if (qflag & 16) {
+                    // copy this lane's query row from the TMA buffer into tensor memory
+                    const int qb = qflag & 1;
+                    const uint32_t u = qb ? qu1 : qu0;
+                    if (active) {
+                        if (!mbar_wait(bar_qfull + 8 * qb, u & 1) ||
+                            !mbar_wait(bar_qtfree + 8 * qb, (u & 1) ^ 1)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint8_t* qrow = sbase + C::OFF_Q + qb * C::QBUF + tl * 128;
+#pragma unroll
+                        for (int h = 0; h < D / 64; ++h) {
+                            uint32_t w[32];
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                const uint4 v = *reinterpret_cast<const uint4*>(
+                                    qrow + h * C::QHALF + ((c ^ (tl & 7)) << 4));
+                                w[4 * c + 0] = v.x; w[4 * c + 1] = v.y;
+                                w[4 * c + 2] = v.z; w[4 * c + 3] = v.w;
+                            }
+                            tmem_st32u(trow + C::Q_COL + qb * (D / 2) + 32 * h, w);
+                        }
+                        tmem_wait_st();
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(bar_qtfull + 8 * qb);
+                        mbar_arrive(bar_qempty + 8 * qb);
+                    }
+                    if (qb) ++qu1; else ++qu0;
+                }
+            }
+            if (flags & kBad) {
+                poison = true;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_pfull + 8 * st);   // meta read: the stage may be reused
+            } else {
+                const int key0 = ma.z + kofs;                // first key of this slice
+                const uint32_t sb = n_qk & 1;
+                if (!mbar_wait(bar_sfull + 8 * sb, (n_qk >> 1) & 1)) { ok = false; break; }
+                tc_fence_after();
+                float sv[KW];
+                if (active) {
+                    if constexpr (KW == 16) {
+                        tmem_ld16(trow + C::S_COL + sb * 64 + kofs, sv);
+                    } else {
+#pragma unroll
+                        for (int h = 0; h < KW / 32; ++h) {
+                            float t[32];
+                            tmem_ld32(trow + C::S_COL + sb * 64 + kofs + 32 * h, t);
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) sv[32 * h + j] = t[j];
+                        }
+                    }
+                    tmem_wait_ld();
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_sfree + 8 * sb);
+                ++n_qk;
+                float factor = 1.f;
+                if (active) {
+                    if (key0 + KW > lim) {
+#pragma unroll
+                        for (int j = 0; j < KW; ++j)
+                            if (key0 + j >= lim) sv[j] = NEG_INF;
+                    }
+                    float mx = NEG_INF;
+#pragma unroll
+                    for (int j = 0; j < KW; ++j) mx = fmaxf(mx, sv[j]);
+                    const float t = mx * sl2;
+                    if (t > m + kLazy) {                  // also true while m is -inf
+                        factor = ex2(m - t);              // 0 when m is -inf
+                        l *= factor;
+                        m = t;
+                    }
+                    const float mr = (m == NEG_INF) ? 0.f : m;
+                    float rs = 0.f;
+#pragma unroll
+                    for (int j = 0; j < KW; ++j) {
+                        sv[j] = ex2(fmaf(sv[j], sl2, -mr));
+                        rs += sv[j];
+                    }
+                    l += rs;
+                }
+                const uint32_t pb = n_pv & 1;
+                if (active) {
+                    // PV two tiles back read this P buffer: it must have completed
+                    if (n_pv >= 2 && !mbar_wait(bar_obar + 8 * pb, ((n_pv - 2) >> 1) & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    if (seg_pv > 0 && __any_sync(0xffffffffu, factor != 1.f)) {
+                        // rescale this row of O in tensor memory once the last PV is done
+                        if (!mbar_wait(bar_obar + 8 * (pb ^ 1), ((n_pv - 1) >> 1) & 1)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            float ov[32];
+                            tmem_ld32(trow + C::O_COL + 32 * c, ov);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) ov[j] *= factor;
+                            tmem_st32(trow + C::O_COL + 32 * c, ov);
+                        }
+                    }
+                    tc_fence_after();
+                    // key 2j of the slice in the low half of its column, 2j+1 in the high half
+                    uint32_t hi[KW / 2], lo[KW / 2];
+#pragma unroll
+                    for (int j = 0; j < KW / 2; ++j) {
+                        const float a = sv[2 * j], b = sv[2 * j + 1];
+                        hi[j] = pack_bf16(a, b);
+                        lo[j] = pack_bf16(a - bf16lo_to_f32(hi[j]), b - bf16hi_to_f32(hi[j]));
+                    }
+                    const uint32_t pc = trow + C::P_COL + pb * 64 + kofs / 2;
+                    if constexpr (KW == 16) {
+                        tmem_st8u(pc, hi);
+                        tmem_st8u(pc + 32, lo);
+                    } else if constexpr (KW == 32) {
+                        tmem_st16u(pc, hi);
+                        tmem_st16u(pc + 32, lo);
+                    } else {
+                        tmem_st32u(pc, *reinterpret_cast<const uint32_t(*)[32]>(hi));
+                        tmem_st32u(pc + 32, *reinterpret_cast<const uint32_t(*)[32]>(lo));
+                    }
+                    tmem_wait_st();
+                }
+                if (ma.z + kPage > leff && tl < kPage && ma.z + tl >= leff) {
+                    // V rows of keys no query may see: their slots may hold anything
+                    uint8_t* const vt = sbase + st * C::STAGE + C::TILE + tl * 128;
+#pragma unroll
+                    for (int h = 0; h < D / 64; ++h)
+#pragma unroll
+                        for (int c = 0; c < 8; ++c)
+                            *reinterpret_cast<uint4*>(vt + h * 8192 + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
+                }
+                fence_proxy_async();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_pfull + 8 * st);
+                ++n_pv;
+                ++seg_pv;
+            }
+            if (flags & kLast) {
+                // ---- segment end: merge the copies, write the output or a partial
+                if (active && seg_pv > 0 &&
+                    !mbar_wait(bar_obar + 8 * ((n_pv - 1) & 1), ((n_pv - 1) >> 1) & 1)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                // weight of this copy: 2^(m_copy - M) with M the max over copies
+                if (NC > 1) {
+                    mls[tl] = make_float2(m, l);
+                    if (!grp_sync()) { ok = false; break; }
+                }
+                float wgt, inv, lse;
+                {
+                    float M = NEG_INF;
+#pragma unroll
+                    for (int c = 0; c < NC; ++c) M = fmaxf(M, NC > 1 ? mls[32 * C::RB * c + r].x : m);
+                    const float Mr = (M == NEG_INF) ? 0.f : M;
+                    float L = 0.f;
+#pragma unroll
+                    for (int c = 0; c < NC; ++c) {
+                        const float2 v = NC > 1 ? mls[32 * C::RB * c + r] : make_float2(m, l);
+                        L += ex2(v.x - Mr) * v.y;
+                    }
+                    wgt = ex2(m - Mr);
+                    inv = (L > 0.f) ? 1.f / L : 0.f;
+                    lse = (L > 0.f) ? M + __log2f(L) : NEG_INF;
+                }
+                const bool nan = poison || seg_pv == 0;
+                float* dst = nullptr;
+                if (copy == 0 && r < p.R)
+                    dst = cur_nseg == 1 ? out_row(p, cur_b, cur_g, r, D)
+                                        : p.part_o + ((long long)cur_slot * p.R + r) * D;
+#pragma unroll 1
+                for (int c = 0; c < D / 32; ++c) {
+                    float ov[32];
+                    if (active) {
+                        tmem_ld32(trow + C::O_COL + 32 * c, ov);
+                        tmem_wait_ld();
+                    }
+                    float* const sc = scr + (c & 1) * C::SCR_ROWS * C::SCR_LD;
+                    if (NC > 1) {
+                        if (copy > 0 && active) {
+                            float* const row = sc + (tl - 32 * C::RB) * C::SCR_LD;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) row[j] = ov[j] * wgt;
+                        }
+                        if (!grp_sync()) { ok = false; break; }
+                    }
+                    if (dst) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            float acc = ov[j] * wgt;
+#pragma unroll
+                            for (int cc = 1; cc < NC; ++cc)
+                                acc += sc[(32 * C::RB * (cc - 1) + r) * C::SCR_LD + j];
+                            ov[j] = acc * inv;
+                        }
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4) {
+                            const float4 v = nan ? make_float4(NANF, NANF, NANF, NANF)
+                                                 : make_float4(ov[j], ov[j + 1], ov[j + 2], ov[j + 3]);
+                            *reinterpret_cast<float4*>(dst + 32 * c + j) = v;
+                        }
+                    }
+                }
+                if (!ok) break;
+                if (dst && cur_nseg > 1) p.part_lse[(long long)cur_slot * p.R + r] = nan ? NANF : lse;
+                tc_fence_before();
+                if (cur_nseg > 1) {
+                    // publish this segment; the CTA completing the pair merges it
+                    __threadfence();
+                    if (!grp_sync()) { ok = false; break; }
+                    if (gtid == 0) {
+                        const int old = atomicAdd(p.cnt + cur_b * p.Hkv + cur_g, 1);
+                        misc[1] = (old == cur_nseg - 1);
+                    }
+                    if (!grp_sync()) { ok = false; break; }
+                    if (misc[1]) {
+                        __threadfence();
+                        merge_pair<D>(p, cur_b, cur_g, cur_nseg, cur_first, gtid, 128);
+                    }
+                }
+            }
+            if (++st == NST) { st = 0; ph ^= 1; }
+        }
+        if (!ok) err |= kErrTimeout;
+    }
+    if (err) atomicOr(&p.err[blockIdx.x], (int)err);
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+}  // namespace spire
