@@ -128,6 +128,35 @@ SPIRE_API spire_status spire_verify_attention(const void *q, const void *k_cache
                                     void *stream);
 
 /*
+ * spire_verify_attention_noalloc -- spire_verify_attention for callers that
+ * cannot allocate device memory at call time (for example a serving engine
+ * that gives all free GPU memory to its KV-cache pool at start-up, or a
+ * plugin host that passes only input and output pointers).  The paper has no
+ * counterpart: this is a property of the library, not of the method.
+ *
+ * Arguments and results are those of spire_verify_attention without the
+ * workspace: its scratch (split partials, arrival counters, error words) is
+ * one file-scope device array of 32 MiB, reserved on every GPU that loads
+ * libspire until the process exits.  Nothing is allocated by the call.
+ *   - A shape whose workspace (spire_verify_workspace_bytes) exceeds 32 MiB
+ *     returns SPIRE_ERR_WORKSPACE; at head_dim 128 that allows up to about 60
+ *     query rows per KV head ((Hq/Hkv)*(k+1)).  Invalid shapes return the same
+ *     status as spire_verify_attention.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - All calls share the one array: calls that may overlap on the GPU (on
+ *     different streams, or from different threads) race and must not be
+ *     issued.  The array keeps the last call's contents; each call clears what
+ *     must start at zero.  spire_get_device_error is not available for it.
+ */
+SPIRE_API spire_status spire_verify_attention_noalloc(const void *q, const void *k_cache,
+                                                      const void *v_cache,
+                                                      const int32_t *block_table,
+                                                      const int32_t *ctx_lens, int32_t k,
+                                                      const spire_attn_desc *desc, float *out,
+                                                      void *stream);
+
+/*
  * spire_draft_workspace_bytes -- workspace size for
  * spire_draft_sparse_attention.  Returns 0 for invalid arguments.
  */

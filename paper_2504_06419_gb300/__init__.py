@@ -21,10 +21,12 @@ import torch
 from . import _lib
 from ._lib import (SpireError, make_desc, spire_draft_slot, spire_draft_sparse_attention,
                    spire_draft_workspace_bytes, spire_get_device_error, spire_status_string,
-                   spire_verify_attention, spire_verify_workspace_bytes)
+                   spire_verify_attention, spire_verify_attention_noalloc,
+                   spire_verify_workspace_bytes)
 
 __all__ = [
-    "SpireError", "make_desc", "spire_verify_attention", "spire_draft_sparse_attention",
+    "SpireError", "make_desc", "spire_verify_attention", "spire_verify_attention_noalloc",
+    "spire_draft_sparse_attention",
     "spire_verify_workspace_bytes", "spire_draft_workspace_bytes", "spire_draft_slot",
     "spire_get_device_error", "spire_status_string", "verify_attention", "draft_attention",
     "verify_desc", "draft_desc",

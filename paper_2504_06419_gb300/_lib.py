@@ -31,6 +31,7 @@ SPIRE_MAX_ROWS_PER_KV_HEAD = 128
 EXPORTED = (
     "spire_verify_workspace_bytes",
     "spire_verify_attention",
+    "spire_verify_attention_noalloc",
     "spire_draft_workspace_bytes",
     "spire_draft_sparse_attention",
     "spire_draft_slot",
@@ -69,6 +70,8 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_verify_workspace_bytes.argtypes = [D, I32]
     lib.spire_verify_attention.restype = ctypes.c_int
     lib.spire_verify_attention.argtypes = [P, P, P, P, P, I32, D, P, P, SZ, P]
+    lib.spire_verify_attention_noalloc.restype = ctypes.c_int
+    lib.spire_verify_attention_noalloc.argtypes = [P, P, P, P, P, I32, D, P, P]
     lib.spire_draft_workspace_bytes.restype = SZ
     lib.spire_draft_workspace_bytes.argtypes = [D, I32, I32]
     lib.spire_draft_sparse_attention.restype = ctypes.c_int
@@ -129,6 +132,15 @@ def spire_verify_attention(q, k_cache, v_cache, block_table, ctx_lens, k, desc, 
     return int(LIB.spire_verify_attention(
         _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(ctx_lens), int(k),
         _desc_ref(desc), _ptr(out), _ptr(workspace), int(ws_bytes), _stream(stream, q)))
+
+
+def spire_verify_attention_noalloc(q, k_cache, v_cache, block_table, ctx_lens, k, desc, out,
+                                   stream=None) -> int:
+    """Verification attention with the library's own fixed scratch (no
+    workspace argument, nothing allocated); see include/spire.h."""
+    return int(LIB.spire_verify_attention_noalloc(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(ctx_lens), int(k),
+        _desc_ref(desc), _ptr(out), _stream(stream, q)))
 
 
 def spire_draft_sparse_attention(q, kv, ctx_lens, n_sink, window, desc, out, workspace, ws_bytes,

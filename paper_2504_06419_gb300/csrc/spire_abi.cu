@@ -302,3 +302,57 @@ const char* spire_status_string(spire_status status) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Verification attention without a caller-provided workspace.
+//
+// Some callers cannot allocate device memory when they call us: a serving
+// engine that hands all free GPU memory to its KV-cache pool at start-up, or a
+// plugin / foreign-function host that passes only input and output pointers
+// and has no CUDA allocator of its own.  For them the split partials, arrival
+// counters and error words live in one file-scope device array of fixed size
+// that every GPU loading this library reserves until the process exits.
+namespace {
+
+constexpr size_t kStaticWsBytes = size_t(32) << 20;   // 32 MiB
+
+static __device__ __align__(256) unsigned char g_static_ws[kStaticWsBytes];
+
+// Device address of g_static_ws on the current device, looked up once per
+// device (cudaGetSymbolAddress, which allocates nothing).
+spire_status static_ws_address(void** out) {
+    static std::mutex mu;
+    static void* addr[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SPIRE_ERR_CUDA;
+    std::lock_guard<std::mutex> g(mu);
+    if (dev >= 0 && dev < 64 && addr[dev]) {
+        *out = addr[dev];
+        return SPIRE_OK;
+    }
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || !p) return SPIRE_ERR_CUDA;
+    if (dev >= 0 && dev < 64) addr[dev] = p;
+    *out = p;
+    return SPIRE_OK;
+}
+
+}  // namespace
+
+extern "C" spire_status spire_verify_attention_noalloc(const void* q, const void* k_cache,
+                                                       const void* v_cache,
+                                                       const int32_t* block_table,
+                                                       const int32_t* ctx_lens, int32_t k,
+                                                       const spire_attn_desc* desc, float* out,
+                                                       void* stream) {
+    const size_t need = spire_verify_workspace_bytes(desc, k);
+    if (need == 0)   // invalid shapes: report them exactly as the workspace entry point does
+        return spire_verify_attention(q, k_cache, v_cache, block_table, ctx_lens, k, desc, out,
+                                      nullptr, 0, stream);
+    if (need > kStaticWsBytes) return SPIRE_ERR_WORKSPACE;
+    void* ws = nullptr;
+    const spire_status st = static_ws_address(&ws);
+    if (st != SPIRE_OK) return st;
+    return spire_verify_attention(q, k_cache, v_cache, block_table, ctx_lens, k, desc, out, ws,
+                                  kStaticWsBytes, stream);
+}

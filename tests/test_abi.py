@@ -27,7 +27,7 @@ def test_header_declares_the_boundary():
     names = declared_functions()
     assert names == sorted([
         "spire_verify_workspace_bytes", "spire_verify_attention",
-        "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
+        "spire_verify_attention_noalloc", "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
         "spire_get_device_error", "spire_status_string"]), names
 
 
