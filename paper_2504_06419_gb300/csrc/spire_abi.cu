@@ -1,6 +1,7 @@
 // spire_abi.cu -- the C ABI of libspire (declared in include/spire.h): host
 // validation, workspace layout, TMA descriptors and the launch on the
-// caller's stream (a memset of the pair counters, then one attention kernel).
+// caller's stream (a small kernel zeroing the pair counters, then one
+// attention kernel that overlaps it through programmatic dependent launch).
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -131,6 +132,13 @@ spire_status device_info(DeviceInfo* out) {
     return SPIRE_OK;
 }
 
+// Zeroes the per-pair arrival counters; lets the attention kernel launched
+// after it start its prologue at once (programmatic dependent launch).
+__global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n) {
+    grid_dep_launch_dependents();
+    for (int i = threadIdx.x; i < n; i += blockDim.x) cnt[i] = 0;
+}
+
 // Shared launch sequence for both calls.
 spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorMap& tv,
                  const int32_t* block_table, const int32_t* ctx_lens, int kp1,
@@ -170,7 +178,8 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     CUtensorMap tq;
     if (!encode_q_map(&tq, q, D, d->num_q_heads, uint64_t(B) * kp1, ap.G, kp1))
         return SPIRE_ERR_CUDA;
-    if (cudaMemsetAsync(ap.cnt, 0, size_t(B) * Hkv * 4, stream) != cudaSuccess) return SPIRE_ERR_CUDA;
+    zero_counters_kernel<<<1, 256, 0, stream>>>(ap.cnt, B * Hkv);
+    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
     const int ctas = di.sms < kMaxCtas ? di.sms : kMaxCtas;
     const int mt = (R + 15) / 16;
     // tcgen05 path when a KV head serves enough query rows to make QK^T and PV

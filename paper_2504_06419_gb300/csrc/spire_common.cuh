@@ -8,10 +8,12 @@
 // query rows per KV head against a run of 64-token K/V tiles.
 //
 // Decomposition.  The unit of work is one 64-token tile of one
-// (sequence b, KV head g) pair.  Pairs are laid end to end in the order
-// (b, g) and their tiles numbered globally 0..W-1.  CTA c of a grid of N
-// takes the contiguous range [floor(cW/N), floor((c+1)W/N)): every SM streams
-// the same number of tiles whatever the spread of lengths.  A pair whose
+// (sequence b, KV head g) pair, plus kHead units of fixed cost per pair (its
+// query load and epilogue).  Pairs are laid end to end in the order (b, g),
+// each as [kHead head units | T tile units], numbered globally 0..W-1.  CTA c
+// of a grid of N takes the contiguous range [floor(cW/N), floor((c+1)W/N)):
+// every SM gets the same work whatever the spread of lengths, counting the
+// per-pair cost that many short pairs add.  A pair whose
 // tiles straddle CTA ranges is computed in segments; each segment leaves a
 // normalised partial (O, log-sum-exp) in a slot of the workspace, and the
 // CTA that finishes a pair's last segment (an arrival counter decides)
@@ -33,6 +35,7 @@ namespace spire {
 
 constexpr int kPage = 64;        // tokens per K/V tile (and per page)
 constexpr int kMaxCtas = 512;    // grid cap; the workspace holds 2 partial slots per CTA
+constexpr int kHead = 4;         // per-pair fixed cost, in tiles (tuned on GB300, ragged lengths)
 
 constexpr uint32_t kErrCtxLen = 1u;
 constexpr uint32_t kErrPageId = 2u;
@@ -135,12 +138,12 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
     for (int b = threadIdx.x; b < p.B; b += blockDim.x) {
         int le;
         bool ok;
-        acc += seq_tiles(p, p.ctx_lens[b], &le, &ok);
+        acc += seq_tiles(p, p.ctx_lens[b], &le, &ok) + kHead;
         bad |= !ok;
     }
-    const long long tiles = block_sum(acc, sh);
+    const long long units = block_sum(acc, sh);
     const int any_bad = __syncthreads_or(bad);
-    const long long W = tiles * p.Hkv;
+    const long long W = units * p.Hkv;
     const int N = W < (long long)gridDim.x ? (int)W : (int)gridDim.x;
     const int c = blockIdx.x;
     const long long lo = c < N ? range_lo(c, W, N) : W, hi = c < N ? range_lo(c + 1, W, N) : W;
@@ -153,10 +156,10 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
         const int b = base + threadIdx.x;
         int le;
         bool ok;
-        const long long T = b < p.B ? seq_tiles(p, p.ctx_lens[b], &le, &ok) : 0;
+        const long long U = b < p.B ? seq_tiles(p, p.ctx_lens[b], &le, &ok) + kHead : 0;
         long long chunk;
-        const long long P = carry + block_excl_scan(T, sh, &chunk);
-        if (b < p.B && lo < hi && P * p.Hkv <= lo && lo < (P + T) * p.Hkv) {
+        const long long P = carry + block_excl_scan(U, sh, &chunk);
+        if (b < p.B && lo < hi && P * p.Hkv <= lo && lo < (P + U) * p.Hkv) {
             sh->b0 = b;
             sh->p0 = P * p.Hkv;
         }
@@ -171,49 +174,56 @@ struct TileMeta {
     int flags, slot, nseg, first_slot;
 };
 
-// Walks this CTA's tile range in order, tracking (b, g, t) incrementally;
-// the segment bookkeeping (divisions) runs once per segment, not per tile.
+// Walks the tiles of this CTA's unit range in order, tracking (b, g, t)
+// incrementally and stepping over head units; the segment bookkeeping
+// (divisions) runs once per segment, not per tile.
 struct TileWalker {
-    long long x, hi, lo, W;    // next tile, end of range, start of range, total
+    long long x, hi, lo, W;    // unit of the next tile, end / start of range, total units
     int N;
     int b, g, t, T, leff;      // current sequence / KV head / tile-in-pair, tiles per pair
-    bool valid;
+    bool valid, first;
     int slot, nseg, first_slot;
 
     __device__ void init(const AttnParams& p, const SchedShared& sh) {
         x = sh.lo; hi = sh.hi; lo = sh.lo; W = sh.W; N = sh.N;
-        b = sh.b0; g = 0; t = 0; T = 1; leff = 0; valid = false;
+        b = sh.b0; g = 0; t = 0; T = 1; leff = 0; valid = false; first = true;
         slot = nseg = first_slot = 0;
         if (x < hi) {
             T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
             const long long off = x - sh.p0;
-            g = (int)(off / T);
-            t = (int)(off - (long long)g * T);
+            const int U = T + kHead;
+            g = (int)(off / U);
+            const int u = (int)(off - (long long)g * U);
+            if (u < kHead) x += kHead - u;         // range starts in a pair's head
+            else t = u - kHead;
         }
     }
     __device__ bool done() const { return x >= hi; }
 
-    // Fills m for tile x and advances; returns the tile index within the pair.
+    // Fills m for the tile at unit x and advances; returns the tile index
+    // within the pair.
     __device__ int next(const AttnParams& p, TileMeta* m) {
         int flags = 0;
-        if (x == lo || t == 0) {
+        if (first || t == 0) {
             flags |= kFirst;
-            // pair_start is the global index of tile 0 of this pair
-            const long long pair_start = x - t, pair_end = pair_start + T;
+            // units of this pair's first / last tile and of its head
+            const long long ftile = x - t, ltile = ftile + T - 1, pstart = ftile - kHead;
             const int c = blockIdx.x;
-            const int c0 = cta_of(pair_start, W, N), c1 = cta_of(pair_end - 1, W, N);
-            slot = (pair_start <= lo) ? 2 * c : 2 * c + 1;   // first segment of this CTA?
+            const int c0 = cta_of(ftile, W, N), c1 = cta_of(ltile, W, N);
+            slot = (lo >= pstart) ? 2 * c : 2 * c + 1;   // first segment of this CTA?
             nseg = c1 - c0 + 1;
-            first_slot = (range_lo(c0, W, N) == pair_start) ? 2 * c0 : 2 * c0 + 1;
+            first_slot = (range_lo(c0, W, N) >= pstart) ? 2 * c0 : 2 * c0 + 1;
         }
         if (x == hi - 1 || t == T - 1) flags |= kLast;
         if (!valid) flags |= kBad;
         m->b = b; m->g = g; m->key0 = t * kPage; m->leff = leff;
         m->flags = flags; m->slot = slot; m->nseg = nseg; m->first_slot = first_slot;
         const int tile = t;
+        first = false;
         ++x;
-        if (++t == T) {
+        if (++t == T) {                            // next pair: step over its head
             t = 0;
+            x += kHead;
             if (++g == p.Hkv) {
                 g = 0;
                 if (x < hi) {

@@ -92,6 +92,8 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         reinterpret_cast<uint4*>(sbase + C::OFF_Q)[i] = make_uint4(0u, 0u, 0u, 0u);
     fence_proxy_async();
     sched_setup(p, sh);   // ends with __syncthreads()
+    // the arrival counters were zeroed by the kernel launched just before
+    grid_dep_wait();
 
     if (warp == C::NW) {
         // ------------------------------------------------------ producer

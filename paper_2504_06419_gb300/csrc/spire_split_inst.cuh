@@ -8,6 +8,26 @@
 
 namespace spire {
 
+// Launch with programmatic stream serialisation: the kernel may start while
+// the counter-zeroing kernel before it finishes, and waits for it
+// (griddepcontrol.wait) before touching the counters.
+template <typename Kern>
+cudaError_t launch_pdl(Kern kern, int ctas, int threads, int smem, cudaStream_t stream,
+                       const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
+                       const AttnParams& p) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(ctas);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, tk, tv, tq, p);
+}
+
 template <int D, int MT>
 cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
                           const AttnParams& p, int ctas, cudaStream_t stream) {
@@ -29,8 +49,7 @@ cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CU
         done.fetch_or(bit, std::memory_order_acq_rel);
     }
     // one CTA per SM: the stage ring takes most of the shared memory
-    kern<<<ctas, C::THREADS, C::SMEM, stream>>>(tk, tv, tq, p);
-    return cudaGetLastError();
+    return launch_pdl(kern, ctas, C::THREADS, C::SMEM, stream, tk, tv, tq, p);
 }
 
 template <int D, int NC>
@@ -51,8 +70,7 @@ cudaError_t launch_tc_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUte
         if (e != cudaSuccess) return e;
         done.fetch_or(bit, std::memory_order_acq_rel);
     }
-    kern<<<ctas, C::THREADS, C::SMEM, stream>>>(tk, tv, tq, p);
-    return cudaGetLastError();
+    return launch_pdl(kern, ctas, C::THREADS, C::SMEM, stream, tk, tv, tq, p);
 }
 
 template <int D>

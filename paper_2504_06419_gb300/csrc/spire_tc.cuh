@@ -35,9 +35,10 @@
 // Tensor memory: S double buffer in columns [0, 128), O in [128, 128 + D),
 // P double buffer in [256, 384) (per buffer: 32 columns of packed P_hi, then
 // 32 of P_lo; key 2j in the low half of column j), Q double buffer in
-// [384, 384 + D) (D/2 packed columns per buffer).  The softmax warps copy each
+// [384, 384 + D) (D/2 packed columns per buffer).  The QK issuer copies each
 // pair's query rows from the TMA buffer in shared memory into tensor memory
-// once per segment, so QK reads only the K tile from shared memory.  Double buffers let the
+// with tcgen05.cp (in order with its MMAs), so QK reads only the K tile from
+// shared memory and the next pair's QK overlaps this pair's epilogue.  Double buffers let the
 // softmax of tile n+1 run while PV of tile n still reads its P.  Every tile,
 // bad or not, is acknowledged on its stage's p_full barrier by the softmax
 // warps and the QK issuer before the PV issuer releases the stage.
@@ -65,7 +66,7 @@ struct TcCfg {
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
     static constexpr int OFF_MISC = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16;
     static constexpr int OFF_BAR = OFF_MISC + 16;
-    static constexpr int NBAR = 3 * NST + 19;
+    static constexpr int NBAR = 3 * NST + 15;
     static constexpr int SMEM = OFF_BAR + NBAR * 8 + 1024;   // + alignment slack
     static constexpr uint32_t TMEM_COLS = 512;
     static constexpr int S_COL = 0, O_COL = 128, P_COL = 256, Q_COL = 384;
@@ -100,7 +101,6 @@ __global__ void __launch_bounds__(224, 1)
     const uint32_t bar_sfull = bar_qempty + 16, bar_sfree = bar_sfull + 16;
     const uint32_t bar_obar = bar_sfree + 16;
     const uint32_t bar_grp = bar_obar + 16, bar_drain = bar_grp + 8;
-    const uint32_t bar_qtfull = bar_drain + 16, bar_qtfree = bar_qtfull + 16;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -111,9 +111,7 @@ __global__ void __launch_bounds__(224, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(bar_qfull + 8 * b, 1);
-            mbar_init(bar_qempty + 8 * b, 4);    // softmax warps copied the rows out
-            mbar_init(bar_qtfull + 8 * b, 4);    // rows are in tensor-memory Q buffer b
-            mbar_init(bar_qtfree + 8 * b, 1);    // the last QK reading it has completed
+            mbar_init(bar_qempty + 8 * b, 1);    // the rows were copied into tensor memory
             mbar_init(bar_sfull + 8 * b, 1);
             mbar_init(bar_sfree + 8 * b, 4);
             mbar_init(bar_obar + 8 * b, 1);    // PV reading P buffer b has completed
@@ -136,6 +134,8 @@ __global__ void __launch_bounds__(224, 1)
     }
     sched_setup(p, sh);   // ends with __syncthreads()
     tc_fence_after();
+    // the arrival counters were zeroed by the kernel launched just before
+    grid_dep_wait();
     const uint32_t tmem = misc[0];
     uint32_t err = 0;
 
@@ -161,10 +161,19 @@ __global__ void __launch_bounds__(224, 1)
                 if (flags & kFirst) {
                     have_q = qflag & 16;
                     if (have_q) {
+                        // the pair's query rows: smem TMA buffer -> tensor-memory buffer qb
                         qb = qflag & 1;
                         const uint32_t par = qb ? cq1 : cq0;
-                        if (!mbar_wait(bar_qtfull + 8 * qb, par)) { ok = false; break; }
+                        if (!mbar_wait(bar_qfull + 8 * qb, par)) { ok = false; break; }
                         if (qb) cq1 ^= 1; else cq0 ^= 1;
+                        tc_fence_after();
+                        const uint32_t qaddr = qsm + qb * C::QBUF;
+#pragma unroll
+                        for (int ks = 0; ks < D / 16; ++ks)
+                            tmem_cp_128x256b(tmem + C::Q_COL + qb * (D / 2) + ks * 8,
+                                             sdesc_sw128(qaddr + (ks >> 2) * C::QHALF + (ks & 3) * 32,
+                                                         16, 1024));
+                        umma_commit(bar_qempty + 8 * qb);   // smem buffer free once copied
                     }
                 }
                 if (!(flags & kBad)) {
@@ -181,7 +190,6 @@ __global__ void __launch_bounds__(224, 1)
                     umma_commit(bar_sfull + 8 * sb);
                     ++n_qk;
                 }
-                if ((flags & kLast) && have_q) umma_commit(bar_qtfree + 8 * qb);
                 mbar_arrive(bar_pfull + 8 * st);   // done with this stage's meta and K tile
                 if (++st == NST) { st = 0; ph ^= 1; }
             }
@@ -248,7 +256,6 @@ __global__ void __launch_bounds__(224, 1)
         const int i_r = min(r / p.G, p.kp1 - 1);      // block row of query row r
         const int kofs = copy * KW;                   // first key of this copy's slice
         uint32_t st = 0, ph = 0, n_qk = 0, n_pv = 0, gph = 0;
-        uint32_t qu0 = 0, qu1 = 0;                    // fills of Q buffer 0 / 1 so far
         float m = NEG_INF, l = 0.f;
         bool poison = false;
         int seg_pv = 0;
@@ -279,41 +286,6 @@ __global__ void __launch_bounds__(224, 1)
                 cur_slot = mb.y; cur_nseg = mb.z; cur_first = mb.w;
                 m = NEG_INF; l = 0.f; poison = false; seg_pv = 0;
                 lim = leff - (p.kp1 - 1) + i_r;
-                const int qflag = mb.x >> 8;
-                if (qflag & 16) {
-                    // copy this lane's query row from the TMA buffer into tensor memory
-                    const int qb = qflag & 1;
-                    const uint32_t u = qb ? qu1 : qu0;
-                    if (active) {
-                        if (!mbar_wait(bar_qfull + 8 * qb, u & 1) ||
-                            !mbar_wait(bar_qtfree + 8 * qb, (u & 1) ^ 1)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint8_t* qrow = sbase + C::OFF_Q + qb * C::QBUF + tl * 128;
-#pragma unroll
-                        for (int h = 0; h < D / 64; ++h) {
-                            uint32_t w[32];
-#pragma unroll
-                            for (int c = 0; c < 8; ++c) {
-                                const uint4 v = *reinterpret_cast<const uint4*>(
-                                    qrow + h * C::QHALF + ((c ^ (tl & 7)) << 4));
-                                w[4 * c + 0] = v.x; w[4 * c + 1] = v.y;
-                                w[4 * c + 2] = v.z; w[4 * c + 3] = v.w;
-                            }
-                            tmem_st32u(trow + C::Q_COL + qb * (D / 2) + 32 * h, w);
-                        }
-                        tmem_wait_st();
-                    }
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) {
-                        mbar_arrive(bar_qtfull + 8 * qb);
-                        mbar_arrive(bar_qempty + 8 * qb);
-                    }
-                    if (qb) ++qu1; else ++qu0;
-                }
             }
             if (flags & kBad) {
                 poison = true;
