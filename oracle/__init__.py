@@ -18,6 +18,9 @@ Functions (each follows the passage cited in ``spire_oracle.c``):
   draft_logical(...)   the same mask over a full-length logical memory
   ring_pack(...)       place logical memory entries into the bounded cache
   draft_slot(p, ...)   slot of logical position p
+  feedback_mix(...)    per-layer feedback memory vectors (Section 3.3)
+  feedback_append(...) memory vector -> K/V projection -> bounded-cache slot
+  round_bf16(v)        nearest-even bf16 bits of a double
 """
 from __future__ import annotations
 
@@ -66,6 +69,13 @@ def _declare(lib):
     lib.oracle_ring_pack.argtypes = [_P, _P, _P, _I32, _I32, _I32, _I64, _I32, _I32, _P]
     lib.oracle_draft_slot.restype = _I64
     lib.oracle_draft_slot.argtypes = [_I64, _I32, _I32]
+    lib.oracle_round_bf16.restype = ctypes.c_uint16
+    lib.oracle_round_bf16.argtypes = [_F64]
+    lib.oracle_feedback_mix.restype = _I64
+    lib.oracle_feedback_mix.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _P]
+    lib.oracle_feedback_append.restype = _I64
+    lib.oracle_feedback_append.argtypes = [_P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32,
+                                           _I32, _I32, _F64, _P]
     return lib
 
 
@@ -191,3 +201,50 @@ def ring_pack(k_log, v_log, ctx_lens, n_sink, window, kv_out=None, lib=None):
 def draft_slot(p, n_sink, window, lib=None):
     lib = lib or load()
     return int(lib.oracle_draft_slot(int(p), int(n_sink), int(window)))
+
+
+def round_bf16(v, lib=None):
+    """Nearest-even bf16 bit pattern of the double v."""
+    lib = lib or load()
+    return int(lib.oracle_round_bf16(float(v)))
+
+
+def feedback_mix(x, w, lib=None):
+    """Memory vectors m [n_dl, B, d_model] (float64) from activations
+    x [n_act, B, d_model] (bf16 bits) and mixing weights w [n_dl, n_act]."""
+    lib = lib or load()
+    x = _u16(x)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    n_act, B, d_model = x.shape
+    n_dl, n_act2 = w.shape
+    if n_act2 != n_act:
+        raise ValueError("w must be [n_dl, n_act]")
+    m = np.zeros((n_dl, B, d_model), dtype=np.float64)
+    if lib.oracle_feedback_mix(_ptr(x), _ptr(w), n_act, n_dl, B, d_model, _ptr(m)) != 0:
+        raise ValueError("oracle_feedback_mix rejected its arguments")
+    return m
+
+
+def feedback_append(x, w, w_kv, pos, kv, n_sink, window, rope_theta=0.0, lib=None):
+    """Append one memory entry per sequence and draft layer to the bounded
+    caches kv [n_dl, B, 2, Hkv, S, D] (bf16 bits, updated in place).
+
+    x [n_act, B, d_model] bf16 bits; w [n_dl, n_act]; w_kv [n_dl, 2*Hkv*D,
+    d_model] bf16 bits; pos int32 [B].  Returns the number of sequences with
+    a negative position (left unwritten)."""
+    lib = lib or load()
+    x, wkv, ps = _u16(x), _u16(w_kv), _i32(pos)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    if not (isinstance(kv, np.ndarray) and kv.dtype == np.uint16 and kv.flags.c_contiguous):
+        raise TypeError("kv must be a C-contiguous uint16 array (updated in place)")
+    n_act, B, d_model = x.shape
+    n_dl, two, Hkv, S, D = kv.shape[0], kv.shape[2], kv.shape[3], kv.shape[4], kv.shape[5]
+    if (kv.shape[1] != B or two != 2 or S != n_sink + window or w.shape != (n_dl, n_act)
+            or wkv.shape != (n_dl, 2 * Hkv * D, d_model) or ps.shape != (B,)):
+        raise ValueError("feedback_append: shape mismatch")
+    n_bad = lib.oracle_feedback_append(_ptr(x), _ptr(w), _ptr(wkv), _ptr(ps), n_act, n_dl, B,
+                                       d_model, Hkv, D, n_sink, window, float(rope_theta),
+                                       _ptr(kv))
+    if n_bad < 0:
+        raise ValueError("oracle_feedback_append rejected its arguments")
+    return int(n_bad)

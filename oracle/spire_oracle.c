@@ -409,3 +409,172 @@ int64_t oracle_ring_pack(const uint16_t *k_log, const uint16_t *v_log,
     }
     return 0;
 }
+
+/* ======================================================================== */
+/* Feedback-memory append (the draft step's cache update)                    */
+/* ======================================================================== */
+/*
+ * After the draft model has run token t, every draft layer i gets a new
+ * memory vector: the softmax(w_i)-weighted average of the token's
+ * activations x_t^0 (embedding) .. x_t^{n_layer} (Section 3.3, the per-layer
+ * memory equation).  Layer i's attention reads keys and values of these
+ * memory vectors, so the vector is projected by the layer's key and value
+ * matrices and the result is stored in the bounded cache at the slot of
+ * logical position p (Section 3.1: sinks plus a sliding window).
+ *
+ * Readings (the paper gives no formula beyond the memory equation):
+ *   - keys and values are plain linear projections of m, no bias, no norm;
+ *   - positional information uses the token's position in the original
+ *     text (Section 3.1, footnote).  When rope_theta > 0 keys are rotated
+ *     by that position with the half-split rotary form: for d < D/2 the
+ *     pair (k[d], k[d + D/2]) is turned by the angle p * rope_theta^(-2d/D);
+ *     values are never rotated;
+ *   - the stored entry is rounded once, to nearest-even bf16.
+ */
+
+/* Round a double to the nearest bf16 (ties to even), returned as bits.
+ * bf16 keeps 8 significant bits; the spacing of bf16 values in
+ * [2^(e-1), 2^e) is 2^(e-8), and below 2^-126 it is fixed at 2^-133. */
+static uint16_t double_to_bf16_bits(double v)
+{
+    if (isnan(v))
+        return 0x7fc0;
+    if (v == 0.0)
+        return signbit(v) ? 0x8000 : 0x0000;
+    int e;
+    frexp(v, &e);                        /* |v| in [2^(e-1), 2^e) */
+    int q = e - 8;
+    if (q < -133)
+        q = -133;
+    double r = ldexp(nearbyint(ldexp(v, -q)), q);   /* exact scaling, RNE */
+    float f = (float)r;                  /* exact: r has <= 8 significant bits */
+    if (fabs(r) > 3.3895313892515355e38) /* beyond the largest finite bf16 */
+        f = r > 0 ? INFINITY : -INFINITY;
+    uint32_t u;
+    memcpy(&u, &f, sizeof(u));
+    return (uint16_t)(u >> 16);
+}
+
+uint16_t oracle_round_bf16(double v)
+{
+    return double_to_bf16_bits(v);
+}
+
+/*
+ * oracle_feedback_mix: m[i, b, :] = sum_l exp(w[i, l]) x[l, b, :] /
+ *                                   sum_l exp(w[i, l]).
+ *   x  bf16 bits [n_act, B, d_model]  (n_act = n_layer + 1, x[0] = embedding)
+ *   w  double [n_dl, n_act]
+ *   m  double [n_dl, B, d_model]
+ * The largest w of each layer is subtracted before exp (the same ratio).
+ */
+int64_t oracle_feedback_mix(const uint16_t *x, const double *w, int32_t n_act,
+                            int32_t n_dl, int32_t B, int32_t d_model, double *m)
+{
+    if (n_act < 1 || n_dl < 1 || B < 0 || d_model < 1)
+        return -1;
+    double *a = (double *)malloc(sizeof(double) * (size_t)n_act);
+    if (!a)
+        return -1;
+    for (int32_t i = 0; i < n_dl; ++i) {
+        double wmax = w[(int64_t)i * n_act];
+        for (int32_t l = 1; l < n_act; ++l)
+            if (w[(int64_t)i * n_act + l] > wmax)
+                wmax = w[(int64_t)i * n_act + l];
+        double z = 0.0;
+        for (int32_t l = 0; l < n_act; ++l) {
+            a[l] = exp(w[(int64_t)i * n_act + l] - wmax);
+            z += a[l];
+        }
+        for (int32_t b = 0; b < B; ++b)
+            for (int32_t c = 0; c < d_model; ++c) {
+                double s = 0.0;
+                for (int32_t l = 0; l < n_act; ++l)
+                    s += a[l] * bf16_to_double(x[((int64_t)l * B + b) * d_model + c]);
+                m[((int64_t)i * B + b) * d_model + c] = s / z;
+            }
+    }
+    free(a);
+    return 0;
+}
+
+/*
+ * oracle_feedback_append: the memory vectors of oracle_feedback_mix, then
+ * for each draft layer i and sequence b
+ *     K[g, d] = sum_c w_kv[i, g*D + d, c]          * m[i, b, c]
+ *     V[g, d] = sum_c w_kv[i, Hkv*D + g*D + d, c]  * m[i, b, c]
+ * rotated (K only, when rope_theta > 0) by position pos[b], rounded to bf16
+ * and written to slot(pos[b]) of layer i's bounded cache.
+ *   w_kv  bf16 bits [n_dl, 2*Hkv*D, d_model]
+ *   pos   int32 [B]: logical position of the new entry (entries before it)
+ *   kv    bf16 bits [n_dl, B, 2, Hkv, n_sink + window, D], updated in place;
+ *         every other slot is left untouched
+ * Returns the number of sequences with pos < 0 (nothing written for them),
+ * or -1 on bad arguments.
+ */
+int64_t oracle_feedback_append(const uint16_t *x, const double *w,
+                               const uint16_t *w_kv, const int32_t *pos,
+                               int32_t n_act, int32_t n_dl, int32_t B,
+                               int32_t d_model, int32_t Hkv, int32_t D,
+                               int32_t n_sink, int32_t window,
+                               double rope_theta, uint16_t *kv)
+{
+    if (n_act < 1 || n_dl < 1 || B < 0 || d_model < 1 || Hkv < 1 || D < 2 ||
+        D % 2 != 0 || n_sink < 0 || window < 1 || rope_theta < 0.0)
+        return -1;
+    if (B == 0)
+        return 0;
+    int64_t S = (int64_t)n_sink + window;
+    int64_t F = 2 * (int64_t)Hkv * D;          /* projected features per layer */
+    double *m = (double *)malloc(sizeof(double) * (size_t)n_dl * B * d_model);
+    double *y = (double *)malloc(sizeof(double) * (size_t)F);
+    if (!m || !y) {
+        free(m);
+        free(y);
+        return -1;
+    }
+    if (oracle_feedback_mix(x, w, n_act, n_dl, B, d_model, m) != 0) {
+        free(m);
+        free(y);
+        return -1;
+    }
+    int64_t n_bad = 0;
+    for (int32_t b = 0; b < B; ++b) {
+        int64_t p = pos[b];
+        if (p < 0) {
+            ++n_bad;
+            continue;
+        }
+        int64_t dst_slot = oracle_draft_slot(p, n_sink, window);
+        for (int32_t i = 0; i < n_dl; ++i) {
+            const double *mi = m + ((int64_t)i * B + b) * d_model;
+            for (int64_t f = 0; f < F; ++f) {
+                const uint16_t *row = w_kv + ((int64_t)i * F + f) * d_model;
+                double acc = 0.0;
+                for (int32_t c = 0; c < d_model; ++c)
+                    acc += bf16_to_double(row[c]) * mi[c];
+                y[f] = acc;
+            }
+            if (rope_theta > 0.0)
+                for (int32_t g = 0; g < Hkv; ++g)
+                    for (int32_t d = 0; d < D / 2; ++d) {
+                        double ang = (double)p * pow(rope_theta, -2.0 * d / D);
+                        double cs = cos(ang), sn = sin(ang);
+                        double *k = y + (int64_t)g * D;
+                        double a0 = k[d], a1 = k[d + D / 2];
+                        k[d] = a0 * cs - a1 * sn;
+                        k[d + D / 2] = a1 * cs + a0 * sn;
+                    }
+            for (int32_t kvi = 0; kvi < 2; ++kvi)
+                for (int32_t g = 0; g < Hkv; ++g) {
+                    uint16_t *dst = kv + (((((int64_t)i * B + b) * 2 + kvi) * Hkv + g) * S + dst_slot) * D;
+                    const double *src = y + ((int64_t)kvi * Hkv + g) * D;
+                    for (int32_t d = 0; d < D; ++d)
+                        dst[d] = double_to_bf16_bits(src[d]);
+                }
+        }
+    }
+    free(m);
+    free(y);
+    return n_bad;
+}

@@ -368,4 +368,183 @@ def pin_draft_invalid_t(lib):
     assert n_bad == 1 and np.all(np.isnan(out[0])) and np.all(np.isfinite(out[1]))
 
 
+
+
+# --------------------------------------------------------------------------
+# feedback-memory append pins
+# --------------------------------------------------------------------------
+def _rand_bf16_bits(rng, shape, scale=1.0):
+    t = torch.from_numpy((rng.standard_normal(shape) * scale).astype(np.float32))
+    return t.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def _torch_round_bf16_bits(v: np.ndarray) -> np.ndarray:
+    """float64 -> float32 -> bf16 (torch, nearest even); double rounding, so
+    it may differ from single rounding by one unit in rare near-tie cases."""
+    t = torch.from_numpy(np.ascontiguousarray(v, dtype=np.float64).astype(np.float32))
+    return t.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def _bf16_ulps(a_bits: np.ndarray, b_bits: np.ndarray) -> np.ndarray:
+    """Distance in bf16 units between two bit arrays (same-sign values)."""
+    def ordered(x):
+        x = x.astype(np.int32)
+        return np.where(x & 0x8000, -(x & 0x7FFF), x)
+    return np.abs(ordered(a_bits) - ordered(b_bits))
+
+
+def pin_round_bf16_ties_and_library(lib):
+    """Nearest-even bf16 rounding: exact ties go to the even neighbour,
+    subnormals and overflow follow IEEE rules, and random float32 values
+    round as torch's float32 -> bf16 conversion does."""
+    ties = {1.0 + 2.0 ** -8: 0x3F80, 1.0 + 3 * 2.0 ** -8: 0x3F82,
+            -(1.0 + 2.0 ** -8): 0xBF80, 2.5 * 2.0 ** -133: 0x0002,
+            3.5 * 2.0 ** -133: 0x0004, 0.5 * 2.0 ** -133: 0x0000,
+            (2 - 2.0 ** -8) * 2.0 ** 127: 0x7F80, 3.0e38: 0x7F62, 0.0: 0x0000}
+    for v, want in ties.items():
+        assert oracle.round_bf16(v, lib=lib) == want, (v, hex(oracle.round_bf16(v, lib=lib)))
+    assert oracle.round_bf16(float("nan"), lib=lib) & 0x7FC0 == 0x7FC0
+    rng = np.random.default_rng(21)
+    vals = np.concatenate([rng.standard_normal(4000) * 10.0 ** rng.integers(-30, 30, 4000),
+                           rng.standard_normal(500) * 1e-39]).astype(np.float32)
+    got = np.array([oracle.round_bf16(float(v), lib=lib) for v in vals], dtype=np.uint16)
+    assert np.array_equal(got, _torch_round_bf16_bits(vals.astype(np.float64)))
+
+
+def pin_feedback_mix_one_hot_and_mean(lib):
+    """w one-hot (one weight 0, the others -1000) gives m = x^l exactly;
+    equal weights give the plain mean over the n_layer + 1 activations."""
+    rng = np.random.default_rng(22)
+    n_act, B, d_model = 3, 5, 64
+    x = _rand_bf16_bits(rng, (n_act, B, d_model))
+    xf = _bits_to_f64(x)
+    w = np.full((n_act + 1, n_act), -1000.0)
+    for i in range(n_act):
+        w[i, i] = 0.0
+    w[n_act] = 0.37
+    m = oracle.feedback_mix(x, w, lib=lib)
+    for i in range(n_act):
+        assert np.array_equal(m[i], xf[i])
+    np.testing.assert_allclose(m[n_act], xf.mean(axis=0), rtol=1e-14, atol=1e-15)
+
+
+def pin_feedback_mix_two_layer_logistic(lib):
+    """Two activations with weights (a, 0): m = s x^0 + (1 - s) x^1 with
+    s = 1 / (1 + e^-a), the logistic function; shifting both weights by a
+    constant changes nothing."""
+    rng = np.random.default_rng(23)
+    x = _rand_bf16_bits(rng, (2, 3, 64))
+    xf = _bits_to_f64(x)
+    for a in (-3.0, 0.0, 0.7, 5.0):
+        s = 1.0 / (1.0 + math.exp(-a))
+        m = oracle.feedback_mix(x, np.array([[a, 0.0], [a + 11.0, 11.0]]), lib=lib)
+        want = s * xf[0] + (1.0 - s) * xf[1]
+        np.testing.assert_allclose(m[0], want, rtol=1e-13, atol=1e-15)
+        np.testing.assert_allclose(m[1], want, rtol=1e-13, atol=1e-15)
+
+
+def _append_case(rng, B, Hkv, D, d_model, n_act, n_dl, n_sink, window):
+    S = n_sink + window
+    x = _rand_bf16_bits(rng, (n_act, B, d_model))
+    w = rng.standard_normal((n_dl, n_act))
+    kv = _rand_bf16_bits(rng, (n_dl, B, 2, Hkv, S, D))
+    return x, w, kv
+
+
+def pin_feedback_append_selection_projection(lib):
+    """With a one-hot mix and a 0/1 selection matrix as the projection, the
+    appended K/V rows are the selected activation entries, bit for bit, in
+    slot(p) of each layer's cache; every other slot is untouched."""
+    rng = np.random.default_rng(24)
+    B, Hkv, D, n_act, n_dl, n_sink, window = 3, 2, 8, 2, 2, 2, 5
+    F = 2 * Hkv * D
+    d_model = F
+    x, _, kv0 = _append_case(rng, B, Hkv, D, d_model, n_act, n_dl, n_sink, window)
+    w = np.array([[0.0, -1000.0], [-1000.0, 0.0]])
+    perms = [rng.permutation(F) for _ in range(n_dl)]
+    wkv = np.zeros((n_dl, F, d_model), dtype=np.float32)
+    for i in range(n_dl):
+        wkv[i, np.arange(F), perms[i]] = 1.0
+    wkv = _f32_to_bf16_bits(wkv)
+    pos = np.array([0, 6, 40], dtype=np.int32)
+    kv = kv0.copy()
+    assert oracle.feedback_append(x, w, wkv, pos, kv, n_sink, window, lib=lib) == 0
+    want = kv0.copy()
+    for i in range(n_dl):
+        for b in range(B):
+            s = oracle.draft_slot(int(pos[b]), n_sink, window, lib=lib)
+            y = x[i, b, perms[i]]
+            want[i, b, 0, :, s] = y[:Hkv * D].reshape(Hkv, D)
+            want[i, b, 1, :, s] = y[Hkv * D:].reshape(Hkv, D)
+    assert np.array_equal(kv, want)
+
+
+def pin_feedback_append_matches_matmul(lib):
+    """Random activations, mixing weights and projections against a float64
+    numpy einsum of the same definition, rounded by torch: every entry within
+    one bf16 unit, nearly all identical (torch rounds twice: via float32)."""
+    rng = np.random.default_rng(25)
+    B, Hkv, D, d_model, n_act, n_dl, n_sink, window = 4, 2, 16, 96, 3, 2, 3, 6
+    x, w, kv0 = _append_case(rng, B, Hkv, D, d_model, n_act, n_dl, n_sink, window)
+    wkv = _rand_bf16_bits(rng, (n_dl, 2 * Hkv * D, d_model), scale=0.1)
+    pos = np.array([1, 9, 2, 30], dtype=np.int32)
+    kv = kv0.copy()
+    oracle.feedback_append(x, w, wkv, pos, kv, n_sink, window, lib=lib)
+    a = np.exp(w - w.max(axis=1, keepdims=True))
+    a /= a.sum(axis=1, keepdims=True)
+    m = np.einsum("il,lbc->ibc", a, _bits_to_f64(x))
+    y = np.einsum("ifc,ibc->ibf", _bits_to_f64(wkv), m)
+    want = _torch_round_bf16_bits(y)
+    got = np.zeros_like(want)
+    for i in range(n_dl):
+        for b in range(B):
+            s = oracle.draft_slot(int(pos[b]), n_sink, window, lib=lib)
+            got[i, b] = kv[i, b, :, :, s].reshape(-1)
+    ulps = _bf16_ulps(got, want)
+    assert ulps.max() <= 1 and (ulps == 0).mean() >= 0.99
+
+
+def pin_feedback_append_rotary_complex_form(lib):
+    """rope_theta > 0 turns each key pair (k[d], k[d + D/2]) by the angle
+    p * theta^(-2d/D): the complex number k[d] + i k[d + D/2] times
+    e^(i angle).  Values are not rotated, position 0 is the identity, and
+    the first and middle frequencies are 1 and theta^-1/2."""
+    rng = np.random.default_rng(26)
+    B, Hkv, D, n_act, n_dl, n_sink, window = 4, 2, 16, 1, 1, 1, 8
+    F = 2 * Hkv * D
+    theta = 10000.0
+    x, _, kv0 = _append_case(rng, B, Hkv, D, F, n_act, n_dl, n_sink, window)
+    w = np.zeros((1, 1))
+    wkv = _f32_to_bf16_bits(np.eye(F, dtype=np.float32)[None])
+    pos = np.array([0, 1, 77, 100003], dtype=np.int32)
+    kv = kv0.copy()
+    oracle.feedback_append(x, w, wkv, pos, kv, n_sink, window, rope_theta=theta, lib=lib)
+    xf = _bits_to_f64(x[0])
+    for b in range(B):
+        s = oracle.draft_slot(int(pos[b]), n_sink, window, lib=lib)
+        kf = xf[b, :Hkv * D].reshape(Hkv, D)
+        assert np.array_equal(kv[0, b, 1, :, s].reshape(-1), x[0, b, Hkv * D:])
+        if pos[b] == 0:
+            assert np.array_equal(kv[0, b, 0, :, s].reshape(-1), x[0, b, :Hkv * D])
+        freq = theta ** (-2.0 * np.arange(D // 2) / D)
+        assert freq[0] == 1.0 and abs(freq[D // 4] - theta ** -0.5) < 1e-15
+        z = (kf[:, :D // 2] + 1j * kf[:, D // 2:]) * np.exp(1j * float(pos[b]) * freq)[None]
+        want = _torch_round_bf16_bits(np.concatenate([z.real, z.imag], axis=1))
+        got = kv[0, b, 0, :, s]
+        ulps = _bf16_ulps(got, want)
+        assert ulps.max() <= 1 and (ulps == 0).mean() >= 0.9
+
+
+def pin_feedback_append_negative_position(lib):
+    """A negative position is counted and writes nothing."""
+    rng = np.random.default_rng(27)
+    x, w, kv0 = _append_case(rng, 2, 1, 8, 16, 2, 1, 1, 4)
+    wkv = _rand_bf16_bits(rng, (1, 16, 16))
+    kv = kv0.copy()
+    n_bad = oracle.feedback_append(x, w, wkv, np.array([-1, 3], dtype=np.int32), kv, 1, 4,
+                                   lib=lib)
+    assert n_bad == 1 and np.array_equal(kv[:, 0], kv0[:, 0])
+    assert not np.array_equal(kv[:, 1], kv0[:, 1])
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

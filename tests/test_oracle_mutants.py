@@ -42,6 +42,23 @@ MUTATIONS = [
      "vals[n] = base + ((((int64_t)b * 2 + 0) * c->Hkv + g) * S + s) * c->D;"),
     ("query_row_stride", "const uint16_t *qi = c->q + (((int64_t)b * rows + i) * c->Hq + h) * c->D;",
      "const uint16_t *qi = c->q + (((int64_t)b * rows) * c->Hq + h) * c->D;"),
+    ("mix_not_normalised", "m[((int64_t)i * B + b) * d_model + c] = s / z;",
+     "m[((int64_t)i * B + b) * d_model + c] = s;"),
+    ("mix_linear_not_exp", "a[l] = exp(w[(int64_t)i * n_act + l] - wmax);",
+     "a[l] = 1.0 + w[(int64_t)i * n_act + l] - wmax;"),
+    ("rope_sign", "k[d] = a0 * cs - a1 * sn;", "k[d] = a0 * cs + a1 * sn;"),
+    ("rope_frequency", "pow(rope_theta, -2.0 * d / D)", "pow(rope_theta, -1.0 * d / D)"),
+    ("rope_adjacent_pairs", "double a0 = k[d], a1 = k[d + D / 2];",
+     "double a0 = k[d], a1 = k[d ^ 1];"),
+    ("append_k_v_swapped", "const double *src = y + ((int64_t)kvi * Hkv + g) * D;",
+     "const double *src = y + ((int64_t)(1 - kvi) * Hkv + g) * D;"),
+    ("append_slot_is_position_mod_s",
+     "int64_t dst_slot = oracle_draft_slot(p, n_sink, window);",
+     "int64_t dst_slot = p % S;"),
+    ("round_truncates", "double r = ldexp(nearbyint(ldexp(v, -q)), q);",
+     "double r = ldexp(trunc(ldexp(v, -q)), q);"),
+    ("round_ties_away", "double r = ldexp(nearbyint(ldexp(v, -q)), q);",
+     "double r = ldexp(round(ldexp(v, -q)), q);"),
 ]
 
 
