@@ -237,9 +237,9 @@ struct TileWalker {
 };
 
 // Shared-memory layout the producer fills: NST stages of [K tile | V tile]
-// (each D/64 boxes of 64 keys x 128 bytes, 128-byte swizzled) and two Q
-// buffers of D/64 halves, each half QHALF bytes of 128-byte rows holding
-// `qcopies` copies of the pair's R query rows, `qcopy_rows` rows apart.
+// (each D/64 boxes of 64 keys x 128 bytes, 128-byte swizzled) and `nqbuf` (1
+// or 2) Q buffers of D/64 halves, each half QHALF bytes of 128-byte rows
+// holding `qcopies` copies of the pair's R query rows, `qcopy_rows` rows apart.
 struct ProducerSmem {
     uint32_t stages;       // shared address of stage 0
     uint32_t q;            // shared address of Q buffer 0
@@ -248,6 +248,7 @@ struct ProducerSmem {
     uint32_t bar_full, bar_empty, bar_qfull, bar_qempty;
     int qcopies;           // copies of the query rows per Q buffer
     int qcopy_rows;        // rows between consecutive copies
+    int nqbuf;             // Q buffers in the ring (1 or 2)
 };
 
 // Meta word layout: meta[2s] = {b, g, key0, leff}; meta[2s+1] = {flags |
@@ -271,7 +272,7 @@ __device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CU
     const uint64_t pol = policy_evict_first();
     const uint32_t qbytes = (D / 64) * sm.qcopies * p.R * 128;
     const uint32_t qbuf = (D / 64) * sm.qhalf;
-    uint32_t st = 0, ph = 0, qs = 0, qph = 0;      // stage ring / Q double buffer
+    uint32_t st = 0, ph = 0, qs = 0, qph = 0;      // stage ring / Q buffer ring
     uint32_t armed = 0, armed_parity = 0;          // stages with a TMA load issued, and its phase
     uint32_t qarmed = 0, qarmed_parity = 0;
     bool ok = true;
@@ -294,7 +295,7 @@ __device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CU
             qarmed |= 1u << qs;
             qarmed_parity = (qarmed_parity & ~(1u << qs)) | (qph << qs);
             qflag = 16 | qs;
-            if (++qs == 2) { qs = 0; qph ^= 1; }
+            if (++qs == (uint32_t)sm.nqbuf) { qs = 0; qph ^= 1; }
         }
         int zk = 0, zv = 0, y = 0;
         if (!(m.flags & kBad)) {
@@ -356,39 +357,74 @@ __device__ __forceinline__ float* out_row(const AttnParams& p, int b, int g, int
 
 // Merge the nseg partials of pair (b, g) into the output; executed by
 // `nthreads` threads with ids 0..nthreads-1.  Partials are read around L1.
+// One pass per output float4: a running maximum M of the segments' base-2
+// log-sum-exps, with the sum and the weighted partial rescaled whenever M
+// grows, so no load waits for another segment's result; each thread handles
+// U outputs per round so that their loads are in flight together.
 template <int D>
 __device__ void merge_pair(const AttnParams& p, int b, int g, int nseg, int first_slot,
                            int tid, int nthreads) {
-    constexpr int D4 = D / 4;
+    constexpr int D4 = D / 4, U = 4;
     const float NEG_INF = __int_as_float(0xff800000);
-    for (int idx = tid; idx < p.R * D4; idx += nthreads) {
-        const int r = idx / D4, d4 = idx - r * D4;
-        float M = NEG_INF;
-        bool nan = false;
+    const float NANF = __int_as_float(0x7fc00000);
+    const int total = p.R * D4;
+    for (int base = tid; base < total; base += U * nthreads) {
+        float M[U], den[U];
+        float4 acc[U];
+        bool nan[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            M[u] = NEG_INF;
+            den[u] = 0.f;
+            acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            nan[u] = false;
+        }
         for (int j = 0; j < nseg; ++j) {
-            const float l = __ldcg(p.part_lse + (long long)segment_slot(j, first_slot) * p.R + r);
-            nan |= (l != l);
-            M = fmaxf(M, l);
+            const long long slot_row = (long long)segment_slot(j, first_slot) * p.R;
+            float lse[U];
+            float4 v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int idx = base + u * nthreads;
+                if (idx < total) {
+                    const int r = idx / D4, d4 = idx - r * D4;
+                    lse[u] = __ldcg(p.part_lse + slot_row + r);
+                    v[u] = __ldcg(reinterpret_cast<const float4*>(p.part_o + (slot_row + r) * D) + d4);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                if (base + u * nthreads >= total) continue;
+                const float l = lse[u];
+                nan[u] |= (l != l);
+                if (l > M[u]) {            // rescale what was accumulated so far
+                    const float sc = ex2(M[u] - l);   // 0 while M is -inf
+                    den[u] *= sc;
+                    acc[u].x *= sc; acc[u].y *= sc; acc[u].z *= sc; acc[u].w *= sc;
+                    M[u] = l;
+                }
+                if (l != NEG_INF && !(l != l)) {
+                    const float w = ex2(l - M[u]);
+                    den[u] += w;
+                    acc[u].x += w * v[u].x; acc[u].y += w * v[u].y;
+                    acc[u].z += w * v[u].z; acc[u].w += w * v[u].w;
+                }
+            }
         }
-        const float Mr = (M == NEG_INF) ? 0.f : M;
-        float den = 0.f;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int j = 0; j < nseg; ++j) {
-            const long long row = (long long)segment_slot(j, first_slot) * p.R + r;
-            const float w = ex2(__ldcg(p.part_lse + row) - Mr);
-            den += w;
-            const float4 v = __ldcg(reinterpret_cast<const float4*>(p.part_o + row * D) + d4);
-            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int idx = base + u * nthreads;
+            if (idx >= total) continue;
+            const int r = idx / D4, d4 = idx - r * D4;
+            float4 res;
+            if (nan[u] || !(den[u] > 0.f)) {
+                res = make_float4(NANF, NANF, NANF, NANF);
+            } else {
+                const float inv = 1.f / den[u];
+                res = make_float4(acc[u].x * inv, acc[u].y * inv, acc[u].z * inv, acc[u].w * inv);
+            }
+            *reinterpret_cast<float4*>(out_row(p, b, g, r, D) + 4 * d4) = res;
         }
-        float4 res;
-        if (nan || !(den > 0.f)) {
-            const float NANF = __int_as_float(0x7fc00000);
-            res = make_float4(NANF, NANF, NANF, NANF);
-        } else {
-            const float inv = 1.f / den;
-            res = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-        }
-        *reinterpret_cast<float4*>(out_row(p, b, g, r, D) + 4 * d4) = res;
     }
 }
 

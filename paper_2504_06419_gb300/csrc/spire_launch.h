@@ -10,9 +10,9 @@
 
 namespace spire {
 
-// Launch the attention kernel for head_dim D with MT m-tiles (16 query rows
-// each) on a grid of `ctas` persistent CTAs.  Returns the launch error, or
-// cudaErrorInvalidValue for an unsupported MT.
+// Launch the warp-MMA attention kernel for head_dim D with MT m-tiles (16
+// query rows each; only MT = 1 is built) on a grid of `ctas` persistent CTAs.
+// Returns the launch error, or cudaErrorInvalidValue for an unsupported MT.
 cudaError_t launch_attn_d64(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tq, const AttnParams& p, int ctas,
                             cudaStream_t stream);
@@ -53,14 +53,13 @@ constexpr int stages() {
     return n > 8 ? 8 : n;
 }
 
-// Deepest stage ring of the tcgen05 kernel next to its two Q buffers and the
-// copy-merge scratch.
+// Deepest stage ring of the tcgen05 kernel next to its Q buffer and the
+// copy-merge scratch: a stage costs its K and V tiles, 32 bytes of tile
+// metadata and three mbarriers.
 template <int D, int NC>
 constexpr int tc_stages() {
-    constexpr int scr = 2 * (NC - 1) * 32 * (4 / NC) * 33 * 4;
-    constexpr int fixed = 2 * (D / 64) * 16384 + scr + 128 * 8 + 8 * 32 + 512 + 16 +
-                          (3 * 8 + 19) * 8 + 1024;
-    constexpr int n = (kMaxDynSmem - fixed) / (2 * 64 * D * 2);
+    constexpr int fixed = TcCfg<D, NC, 0>::SMEM;
+    constexpr int n = (kMaxDynSmem - fixed) / (2 * 64 * D * 2 + 32 + 3 * 8);
     return n > 6 ? 6 : n;
 }
 

@@ -99,7 +99,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         // ------------------------------------------------------ producer
         if (lane != 0) return;
         const ProducerSmem psm{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
-                               bar_empty, bar_qfull, bar_qempty, 1, 0};
+                               bar_empty, bar_qfull, bar_qempty, 1, 0, 2};
         const uint32_t err = produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, psm);
         if (err) atomicOr(&p.err[blockIdx.x], (int)err);
         return;

@@ -89,17 +89,9 @@ template <int D>
 cudaError_t launch_attn_dispatch(int mt, const CUtensorMap& tk, const CUtensorMap& tv,
                                  const CUtensorMap& tq, const AttnParams& p, int ctas,
                                  cudaStream_t stream) {
-    switch (mt) {
-        case 1: return launch_attn_t<D, 1>(tk, tv, tq, p, ctas, stream);
-        case 2: return launch_attn_t<D, 2>(tk, tv, tq, p, ctas, stream);
-        case 3: return launch_attn_t<D, 3>(tk, tv, tq, p, ctas, stream);
-        case 4: return launch_attn_t<D, 4>(tk, tv, tq, p, ctas, stream);
-        case 5: return launch_attn_t<D, 5>(tk, tv, tq, p, ctas, stream);
-        case 6: return launch_attn_t<D, 6>(tk, tv, tq, p, ctas, stream);
-        case 7: return launch_attn_t<D, 7>(tk, tv, tq, p, ctas, stream);
-        case 8: return launch_attn_t<D, 8>(tk, tv, tq, p, ctas, stream);
-        default: return cudaErrorInvalidValue;
-    }
+    // the library sends only pairs of at most 16 query rows (one m-tile) here
+    if (mt != 1) return cudaErrorInvalidValue;
+    return launch_attn_t<D, 1>(tk, tv, tq, p, ctas, stream);
 }
 
 }  // namespace spire

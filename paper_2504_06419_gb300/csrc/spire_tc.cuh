@@ -60,7 +60,7 @@ struct TcCfg {
     static constexpr int SCR_ROWS = (NC - 1) * 32 * RB;   // rows of copies 1 .. NC-1
     static constexpr int SCR_LD = 33;              // floats per scratch row (32 + pad)
     static constexpr int OFF_Q = NST * STAGE;
-    static constexpr int OFF_SCR = OFF_Q + 2 * QBUF;
+    static constexpr int OFF_SCR = OFF_Q + QBUF;   // one Q buffer: copied to TMEM at once
     static constexpr int OFF_ML = OFF_SCR + 2 * SCR_ROWS * SCR_LD * 4;
     static constexpr int OFF_META = OFF_ML + 128 * 8;
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
@@ -124,7 +124,7 @@ __global__ void __launch_bounds__(224, 1)
         p.err[blockIdx.x] = 0;
     }
     // Q rows of padding stay zero for the whole kernel
-    for (int i = threadIdx.x; i < (2 * C::QBUF) / 16; i += blockDim.x)
+    for (int i = threadIdx.x; i < C::QBUF / 16; i += blockDim.x)
         reinterpret_cast<uint4*>(sbase + C::OFF_Q)[i] = make_uint4(0u, 0u, 0u, 0u);
     fence_proxy_async();
     if (warp == 1) {
@@ -143,15 +143,15 @@ __global__ void __launch_bounds__(224, 1)
         // ------------------------------------------------------ producer
         if (lane == 0) {
             const ProducerSmem ps{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
-                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC};
+                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC, 1};
             err |= produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------ QK issuer
         if (lane == 0) {
             constexpr uint32_t ID_QK = idesc_bf16(128, 64, false);
-            uint32_t st = 0, ph = 0, cq0 = 0, cq1 = 0, n_qk = 0;
-            int qb = 0;
+            uint32_t st = 0, ph = 0, cq = 0, n_qk = 0;
+            int qb = 1;                       // tensor-memory Q buffer of the current segment
             bool have_q = false, ok = true;
             for (;;) {
                 if (!mbar_wait(bar_full + 8 * st, ph)) { ok = false; break; }
@@ -161,19 +161,20 @@ __global__ void __launch_bounds__(224, 1)
                 if (flags & kFirst) {
                     have_q = qflag & 16;
                     if (have_q) {
-                        // the pair's query rows: smem TMA buffer -> tensor-memory buffer qb
-                        qb = qflag & 1;
-                        const uint32_t par = qb ? cq1 : cq0;
-                        if (!mbar_wait(bar_qfull + 8 * qb, par)) { ok = false; break; }
-                        if (qb) cq1 ^= 1; else cq0 ^= 1;
+                        // the pair's query rows: the smem TMA buffer -> tensor-memory
+                        // buffer qb (two, alternating, so this copy never overwrites
+                        // rows that QKs of the previous segment may still read)
+                        qb ^= 1;
+                        if (!mbar_wait(bar_qfull, cq)) { ok = false; break; }
+                        cq ^= 1;
                         tc_fence_after();
-                        const uint32_t qaddr = qsm + qb * C::QBUF;
+                        const uint32_t qaddr = qsm;
 #pragma unroll
                         for (int ks = 0; ks < D / 16; ++ks)
                             tmem_cp_128x256b(tmem + C::Q_COL + qb * (D / 2) + ks * 8,
                                              sdesc_sw128(qaddr + (ks >> 2) * C::QHALF + (ks & 3) * 32,
                                                          16, 1024));
-                        umma_commit(bar_qempty + 8 * qb);   // smem buffer free once copied
+                        umma_commit(bar_qempty);   // smem buffer free once copied
                     }
                 }
                 if (!(flags & kBad)) {
@@ -322,9 +323,20 @@ __global__ void __launch_bounds__(224, 1)
                         for (int j = 0; j < KW; ++j)
                             if (key0 + j >= lim) sv[j] = NEG_INF;
                     }
-                    float mx = NEG_INF;
+                    // independent partial maxima (three-input max) keep the chain short
+                    constexpr int NP = KW / 8;        // partials of 8 scores each
+                    float mp[NP];
 #pragma unroll
-                    for (int j = 0; j < KW; ++j) mx = fmaxf(mx, sv[j]);
+                    for (int j = 0; j < NP; ++j) {
+                        const float* v = sv + 8 * j;
+                        mp[j] = fmaxf(fmax3(fmax3(v[0], v[1], v[2]), v[3], v[4]),
+                                      fmax3(v[5], v[6], v[7]));
+                    }
+#pragma unroll
+                    for (int w = NP / 2; w > 0; w /= 2)
+#pragma unroll
+                        for (int j = 0; j < w; ++j) mp[j] = fmaxf(mp[j], mp[j + w]);
+                    const float mx = mp[0];
                     const float t = mx * sl2;
                     if (t > m + kLazy) {                  // also true while m is -inf
                         factor = ex2(m - t);              // 0 when m is -inf
@@ -332,13 +344,24 @@ __global__ void __launch_bounds__(224, 1)
                         m = t;
                     }
                     const float mr = (m == NEG_INF) ? 0.f : m;
-                    float rs = 0.f;
+                    // exponent arguments and partial sums two lanes at a time
+                    const uint64_t scale2 = f2_pack(sl2, sl2), shift2 = f2_pack(-mr, -mr);
+                    uint64_t sp[4];
 #pragma unroll
-                    for (int j = 0; j < KW; ++j) {
-                        sv[j] = ex2(fmaf(sv[j], sl2, -mr));
-                        rs += sv[j];
+                    for (int j = 0; j < 4; ++j) sp[j] = 0ull;
+#pragma unroll
+                    for (int j = 0; j < KW / 2; ++j) {
+                        float x, y;
+                        f2_unpack(fma2(f2_pack(sv[2 * j], sv[2 * j + 1]), scale2, shift2), x, y);
+                        sv[2 * j] = ex2(x);
+                        sv[2 * j + 1] = ex2(y);
+                        sp[j & 3] = add2(sp[j & 3], f2_pack(sv[2 * j], sv[2 * j + 1]));
                     }
-                    l += rs;
+                    {
+                        float x, y;
+                        f2_unpack(add2(add2(sp[0], sp[1]), add2(sp[2], sp[3])), x, y);
+                        l += x + y;
+                    }
                 }
                 const uint32_t pb = n_pv & 1;
                 if (active) {
@@ -347,8 +370,36 @@ __global__ void __launch_bounds__(224, 1)
                         ok = false;
                         break;
                     }
+                    tc_fence_after();
+                    // key 2j of the slice in the low half of its column, 2j+1 in the high
+                    // half; packed and stored 16 or 32 keys at a time
+                    constexpr int PK = KW < 32 ? KW : 32;
+                    const uint32_t pc = trow + C::P_COL + pb * 64 + kofs / 2;
+#pragma unroll
+                    for (int h = 0; h < KW / PK; ++h) {
+                        uint32_t hi[PK / 2], lo[PK / 2];
+#pragma unroll
+                        for (int j = 0; j < PK / 2; ++j) {
+                            const float a = sv[PK * h + 2 * j], b = sv[PK * h + 2 * j + 1];
+                            hi[j] = pack_bf16(a, b);
+                            float ra, rb;   // the parts bf16 rounding dropped
+                            f2_unpack(sub2(f2_pack(a, b), f2_pack(bf16lo_to_f32(hi[j]), bf16hi_to_f32(hi[j]))),
+                                      ra, rb);
+                            lo[j] = pack_bf16(ra, rb);
+                        }
+                        if constexpr (PK == 16) {
+                            tmem_st8u(pc + 8 * h, hi);
+                            tmem_st8u(pc + 32 + 8 * h, lo);
+                        } else {
+                            tmem_st16u(pc + 16 * h, hi);
+                            tmem_st16u(pc + 32 + 16 * h, lo);
+                        }
+                    }
+                    tmem_wait_st();
                     if (seg_pv > 0 && __any_sync(0xffffffffu, factor != 1.f)) {
-                        // rescale this row of O in tensor memory once the last PV is done
+                        // rescale this row of O in tensor memory once the last PV is done;
+                        // after the P store, so the exponentials are no longer live (PV of
+                        // this tile waits for p_full, signalled after this)
                         if (!mbar_wait(bar_obar + 8 * (pb ^ 1), ((n_pv - 1) >> 1) & 1)) {
                             ok = false;
                             break;
@@ -363,28 +414,8 @@ __global__ void __launch_bounds__(224, 1)
                             for (int j = 0; j < 32; ++j) ov[j] *= factor;
                             tmem_st32(trow + C::O_COL + 32 * c, ov);
                         }
+                        tmem_wait_st();
                     }
-                    tc_fence_after();
-                    // key 2j of the slice in the low half of its column, 2j+1 in the high half
-                    uint32_t hi[KW / 2], lo[KW / 2];
-#pragma unroll
-                    for (int j = 0; j < KW / 2; ++j) {
-                        const float a = sv[2 * j], b = sv[2 * j + 1];
-                        hi[j] = pack_bf16(a, b);
-                        lo[j] = pack_bf16(a - bf16lo_to_f32(hi[j]), b - bf16hi_to_f32(hi[j]));
-                    }
-                    const uint32_t pc = trow + C::P_COL + pb * 64 + kofs / 2;
-                    if constexpr (KW == 16) {
-                        tmem_st8u(pc, hi);
-                        tmem_st8u(pc + 32, lo);
-                    } else if constexpr (KW == 32) {
-                        tmem_st16u(pc, hi);
-                        tmem_st16u(pc + 32, lo);
-                    } else {
-                        tmem_st32u(pc, *reinterpret_cast<const uint32_t(*)[32]>(hi));
-                        tmem_st32u(pc + 32, *reinterpret_cast<const uint32_t(*)[32]>(lo));
-                    }
-                    tmem_wait_st();
                 }
                 if (ma.z + kPage > leff && tl < kPage && ma.z + tl >= leff) {
                     // V rows of keys no query may see: their slots may hold anything
@@ -394,8 +425,8 @@ __global__ void __launch_bounds__(224, 1)
 #pragma unroll
                         for (int c = 0; c < 8; ++c)
                             *reinterpret_cast<uint4*>(vt + h * 8192 + 16 * c) = make_uint4(0u, 0u, 0u, 0u);
+                    fence_proxy_async();   // the zeros before the tensor core reads V
                 }
-                fence_proxy_async();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_pfull + 8 * st);
