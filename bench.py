@@ -258,6 +258,8 @@ def spire_arm(args, cfg):
 
     k, Hq, Hkv, D = cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
     L = wl.sample_ctx_lens(cfg)
+    if args.max_seqs:
+        L = L[:args.max_seqs]     # a smaller case of the same workload (profiling captures)
     vi = wl.make_verify(L, k, Hq, Hkv, D, seed=cfg.seed, device=dev, shuffle=cfg.paged_shuffle)
     drafts = [wl.make_draft(wl.draft_ctx_for_step(L, k, j), Hq, Hkv, D, cfg.n_sink, cfg.window,
                             seed=cfg.seed + 17 * (j + 1), device=dev) for j in range(k)]
@@ -358,7 +360,7 @@ def spire_arm(args, cfg):
     ms, eager_ms, v_ms, d_ms = reduce_max([ms, eager_ms, v_ms, d_ms], dist, dev)
     del graph
 
-    B = cfg.batch
+    B = int(L.size)
     tokens = B * (k + 1)
     value = job_value(tokens, world, ms)
     vb = verify_bytes(L, k, Hq, Hkv, D)
@@ -474,6 +476,9 @@ def main():
     ap.add_argument("--config", default="uniform8k", choices=sorted(wl.CONFIGS))
     ap.add_argument("--impl", default="spire", choices=["spire", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--max-seqs", type=int, default=0,
+                    help="use only the first N sequences of the workload (small profiling "
+                         "captures; not a benchmark configuration)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
