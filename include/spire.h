@@ -17,6 +17,10 @@
  *                                 entries plus a sliding window of feedback-
  *                                 memory entries m_{<t} (Sections 3.1, 3.3),
  *                                 over a bounded cache.
+ *   spire_feedback_append         the draft step's cache update: mix the
+ *                                 token's activations into each layer's memory
+ *                                 vector, project it to K/V and store it in
+ *                                 the bounded cache (Section 3.3).
  *
  * Conventions common to every call
  *   - All tensor arguments are DEVICE pointers, owned by the caller; the
@@ -191,6 +195,70 @@ SPIRE_API spire_status spire_draft_sparse_attention(const void *q, const void *k
                                           const spire_attn_desc *desc,
                                           float *out, void *workspace,
                                           size_t ws_bytes, void *stream);
+
+/*
+ * Draft-step cache update: the feedback-memory append.
+ *
+ * After the draft model has run token t, each of its layers i gets a new
+ * memory vector m_t^i, the softmax(w_i)-weighted average of the token's
+ * activations x_t^0 (embedding) .. x_t^{n_layer} (Section 3.3, the per-layer
+ * memory equation; layers share neither memory vectors nor projections).
+ * Layer i attends to keys and values of its memory entries, so the vector is
+ * projected by the layer's key and value matrices and stored in slot
+ * spire_draft_slot(p) of the layer's bounded cache (Section 3.1), where p is
+ * the number of entries before it.  The paper names no positional scheme,
+ * only that SPIRe uses the token's original-text position (Section 3.1,
+ * footnote); with rope_theta > 0 keys are turned by that position (rotary,
+ * half-split pairs (d, d + D/2), angle p * rope_theta^(-2d/D)).
+ */
+typedef struct spire_append_desc {
+    int32_t batch;            /* B >= 1 sequences, one new entry each */
+    int32_t num_act;          /* n_layer + 1 activations mixed (1..16), x^0 = embedding */
+    int32_t num_draft_layers; /* n_dl (1..16): memory vector, projection and cache per layer */
+    int32_t d_model;          /* activation width, a multiple of 64 (64..65536) */
+    int32_t num_kv_heads;     /* Hkv >= 1 */
+    int32_t head_dim;         /* D: 64 or 128 */
+    int32_t n_sink;           /* >= 0 sink slots of each cache */
+    int32_t window;           /* >= 1 window slots of each cache */
+    float rope_theta;         /* > 0: rotate keys by position; 0: no rotation */
+} spire_append_desc;
+
+/*
+ * spire_feedback_append_workspace_bytes -- workspace size for
+ * spire_feedback_append (split-K partials and the device error word).
+ * Returns 0 for invalid arguments.
+ */
+SPIRE_API size_t spire_feedback_append_workspace_bytes(const spire_append_desc *desc);
+
+/*
+ * spire_feedback_append -- write one memory entry per sequence into every
+ * draft layer's bounded cache:
+ *     m[i, b]      = sum_l softmax(mix_w[i, :])_l * x[l, b, :]
+ *     K[i, b, g, :] = w_kv[i, g*D .. g*D + D - 1, :]               . m[i, b]
+ *     V[i, b, g, :] = w_kv[i, Hkv*D + g*D .. Hkv*D + g*D + D - 1, :] . m[i, b]
+ * K rotated by pos[b] when rope_theta > 0, both rounded to nearest-even bf16
+ * and stored at kv[i, b, 0 (K) / 1 (V), g, spire_draft_slot(pos[b]), :].
+ *
+ *   x        bf16 [num_act, B, d_model]: the token's activations.
+ *   mix_w    fp32 [n_dl, num_act]: the learnable weights w_{il}, un-normalised.
+ *   w_kv     bf16 [n_dl, 2*Hkv*D, d_model]: per layer the key rows, then the
+ *            value rows (row-major, d_model contiguous).
+ *   pos      int32 [B] on the device: p >= 0, the entry's logical position.
+ *   kv       bf16 [n_dl, B, 2, Hkv, n_sink + window, D]: the caches (layer i's
+ *            cache is the [B, 2, Hkv, S, D] block spire_draft_sparse_attention
+ *            reads), updated in place; no other slot is written.
+ *   workspace >= spire_feedback_append_workspace_bytes(desc) bytes.
+ * The product runs on the tensor cores with the memory vector split into two
+ * bf16 parts (about 16 significant bits) and fp32 accumulation, so an entry is
+ * within one bf16 unit of the exactly rounded value.  A sequence with
+ * pos[b] < 0 is not written and sets SPIRE_DEVERR_CTX_LEN.  Pointers x, w_kv
+ * and kv must be 16-byte aligned, the workspace 256-byte aligned.
+ */
+SPIRE_API spire_status spire_feedback_append(const void *x, const float *mix_w,
+                                             const void *w_kv, const int32_t *pos,
+                                             const spire_append_desc *desc, void *kv,
+                                             void *workspace, size_t ws_bytes,
+                                             void *stream);
 
 /*
  * spire_draft_slot -- slot of logical memory position p >= 0 in the bounded

@@ -10,6 +10,9 @@ libspire (include/spire.h):
                                  bf16 KV with GQA, causal within the block
   spire_draft_sparse_attention   draft sink + sliding-window attention over a
                                  bounded feedback-memory cache (Section 3.3)
+  spire_feedback_append          the draft step's cache update: per-layer
+                                 memory vector, K/V projection, bounded-cache
+                                 slot (Section 3.3)
 
 The functions below allocate outputs and workspaces with PyTorch and call the
 C ABI; all computation runs in the library's kernels.
@@ -19,14 +22,16 @@ from __future__ import annotations
 import torch
 
 from . import _lib
-from ._lib import (SpireError, make_desc, spire_draft_slot, spire_draft_sparse_attention,
-                   spire_draft_workspace_bytes, spire_get_device_error, spire_status_string,
-                   spire_verify_attention, spire_verify_attention_noalloc,
-                   spire_verify_workspace_bytes)
+from ._lib import (SpireError, make_append_desc, make_desc, spire_draft_slot,
+                   spire_draft_sparse_attention, spire_draft_workspace_bytes,
+                   spire_feedback_append, spire_feedback_append_workspace_bytes,
+                   spire_get_device_error, spire_status_string, spire_verify_attention,
+                   spire_verify_attention_noalloc, spire_verify_workspace_bytes)
 
 __all__ = [
-    "SpireError", "make_desc", "spire_verify_attention", "spire_verify_attention_noalloc",
-    "spire_draft_sparse_attention",
+    "SpireError", "make_desc", "make_append_desc", "spire_verify_attention",
+    "spire_verify_attention_noalloc", "spire_draft_sparse_attention", "spire_feedback_append",
+    "spire_feedback_append_workspace_bytes", "feedback_append",
     "spire_verify_workspace_bytes", "spire_draft_workspace_bytes", "spire_draft_slot",
     "spire_get_device_error", "spire_status_string", "verify_attention", "draft_attention",
     "verify_desc", "draft_desc",
@@ -74,3 +79,25 @@ def draft_attention(q, kv, ctx_lens, n_sink, window, softmax_scale=1.0, out=None
     if st != 0:
         raise SpireError(st, "spire_draft_sparse_attention")
     return out
+
+
+def feedback_append(x, mix_w, w_kv, pos, kv, n_sink, window, rope_theta=0.0, workspace=None,
+                    stream=None):
+    """Write one feedback-memory entry per sequence into every draft layer's
+    bounded cache kv [n_dl, B, 2, Hkv, n_sink + window, D] (bf16, in place).
+
+    x [n_act, B, d_model] bf16, mix_w [n_dl, n_act] fp32, w_kv [n_dl, 2*Hkv*D,
+    d_model] bf16, pos [B] int32 (device).  Returns kv."""
+    n_act, B, d_model = x.shape
+    n_dl, Hkv, D = kv.shape[0], kv.shape[3], kv.shape[5]
+    desc = make_append_desc(B, n_act, n_dl, d_model, Hkv, D, n_sink, window, rope_theta)
+    ws_bytes = spire_feedback_append_workspace_bytes(desc)
+    if ws_bytes == 0:
+        raise SpireError(1, "spire_feedback_append_workspace_bytes")
+    if workspace is None:
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=x.device)
+    st = spire_feedback_append(x, mix_w, w_kv, pos, desc, kv, workspace, workspace.numel(),
+                               stream)
+    if st != 0:
+        raise SpireError(st, "spire_feedback_append")
+    return kv

@@ -34,6 +34,8 @@ EXPORTED = (
     "spire_verify_attention_noalloc",
     "spire_draft_workspace_bytes",
     "spire_draft_sparse_attention",
+    "spire_feedback_append_workspace_bytes",
+    "spire_feedback_append",
     "spire_draft_slot",
     "spire_get_device_error",
     "spire_status_string",
@@ -50,6 +52,20 @@ class spire_attn_desc(ctypes.Structure):
         ("max_pages_per_seq", ctypes.c_int32),
         ("num_pages", ctypes.c_int32),
         ("softmax_scale", ctypes.c_float),
+    ]
+
+
+class spire_append_desc(ctypes.Structure):
+    _fields_ = [
+        ("batch", ctypes.c_int32),
+        ("num_act", ctypes.c_int32),
+        ("num_draft_layers", ctypes.c_int32),
+        ("d_model", ctypes.c_int32),
+        ("num_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("n_sink", ctypes.c_int32),
+        ("window", ctypes.c_int32),
+        ("rope_theta", ctypes.c_float),
     ]
 
 
@@ -76,6 +92,11 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_draft_workspace_bytes.argtypes = [D, I32, I32]
     lib.spire_draft_sparse_attention.restype = ctypes.c_int
     lib.spire_draft_sparse_attention.argtypes = [P, P, P, I32, I32, D, P, P, SZ, P]
+    A = ctypes.POINTER(spire_append_desc)
+    lib.spire_feedback_append_workspace_bytes.restype = SZ
+    lib.spire_feedback_append_workspace_bytes.argtypes = [A]
+    lib.spire_feedback_append.restype = ctypes.c_int
+    lib.spire_feedback_append.argtypes = [P, P, P, P, A, P, P, SZ, P]
     lib.spire_draft_slot.restype = I64
     lib.spire_draft_slot.argtypes = [I64, I32, I32]
     lib.spire_get_device_error.restype = ctypes.c_int
@@ -148,6 +169,23 @@ def spire_draft_sparse_attention(q, kv, ctx_lens, n_sink, window, desc, out, wor
     return int(LIB.spire_draft_sparse_attention(
         _ptr(q), _ptr(kv), _ptr(ctx_lens), int(n_sink), int(window), _desc_ref(desc),
         _ptr(out), _ptr(workspace), int(ws_bytes), _stream(stream, q)))
+
+
+def make_append_desc(batch, num_act, num_draft_layers, d_model, num_kv_heads, head_dim, n_sink,
+                     window, rope_theta=0.0) -> spire_append_desc:
+    return spire_append_desc(int(batch), int(num_act), int(num_draft_layers), int(d_model),
+                             int(num_kv_heads), int(head_dim), int(n_sink), int(window),
+                             float(rope_theta))
+
+
+def spire_feedback_append_workspace_bytes(desc: spire_append_desc) -> int:
+    return int(LIB.spire_feedback_append_workspace_bytes(_desc_ref(desc)))
+
+
+def spire_feedback_append(x, mix_w, w_kv, pos, desc, kv, workspace, ws_bytes, stream=None) -> int:
+    return int(LIB.spire_feedback_append(
+        _ptr(x), _ptr(mix_w), _ptr(w_kv), _ptr(pos), _desc_ref(desc), _ptr(kv), _ptr(workspace),
+        int(ws_bytes), _stream(stream, x)))
 
 
 def spire_draft_slot(pos: int, n_sink: int, window: int) -> int:

@@ -20,7 +20,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libspire.so")
-SOURCES = ["spire_abi.cu", "spire_split_d64.cu", "spire_split_d128.cu"]
+SOURCES = ["spire_abi.cu", "spire_split_d64.cu", "spire_split_d128.cu", "spire_append.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

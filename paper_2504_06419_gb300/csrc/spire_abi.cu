@@ -12,6 +12,7 @@
 #include <cudaTypedefs.h>
 
 #include "spire.h"
+#include "spire_host.h"
 #include "spire_launch.h"
 
 namespace spire {
@@ -131,6 +132,35 @@ spire_status device_info(DeviceInfo* out) {
         return SPIRE_ERR_CUDA;
     return SPIRE_OK;
 }
+
+}  // namespace
+
+bool host_aligned(const void* p, uintptr_t a) { return aligned(p, a); }
+
+spire_status host_device_info(int* sms, int* smem_optin) {
+    DeviceInfo di;
+    const spire_status st = device_info(&di);
+    if (st != SPIRE_OK) return st;
+    *sms = di.sms;
+    *smem_optin = di.smem_optin;
+    return SPIRE_OK;
+}
+
+bool encode_2d_bf16_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                        uint32_t box_inner, uint32_t box_outer) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {inner * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+namespace {
 
 // Zeroes the per-pair arrival counters; lets the attention kernel launched
 // after it start its prologue at once (programmatic dependent launch).

@@ -28,6 +28,7 @@ def test_header_declares_the_boundary():
     assert names == sorted([
         "spire_verify_workspace_bytes", "spire_verify_attention",
         "spire_verify_attention_noalloc", "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
+        "spire_feedback_append_workspace_bytes", "spire_feedback_append",
         "spire_get_device_error", "spire_status_string"]), names
 
 
@@ -120,3 +121,55 @@ def test_workspace_sizes_depend_only_on_shapes(spire):
                                                     num_kv_heads=8, num_pages=10 ** 6), 4) == a
     assert spire.spire_draft_workspace_bytes(d, 16, 512) == spire.spire_draft_workspace_bytes(d, 0, 9)
     assert spire.spire_verify_workspace_bytes(None, 4) == 0
+
+
+def _adesc(spire, **kw):
+    d = dict(batch=64, num_act=3, num_draft_layers=2, d_model=4096, num_kv_heads=8, head_dim=128,
+             n_sink=16, window=512, rope_theta=10000.0)
+    d.update(kw)
+    return spire.make_append_desc(**d)
+
+
+def test_append_workspace_depends_only_on_shapes(spire):
+    d = _adesc(spire)
+    n = spire.spire_feedback_append_workspace_bytes(d)
+    # header + up to 8 K splits x n_dl x B x 2*Hkv*D fp32 partials
+    assert n == 512 + 8 * 2 * 64 * 2048 * 4
+    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, batch=300)) == \
+        512 + 4 * 2 * 300 * 2048 * 4     # 2 token blocks (N = 256): 64 tiles, <= 4 splits
+    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire)) == n
+
+
+@pytest.mark.parametrize("kw", [
+    dict(batch=0), dict(num_act=0), dict(num_act=17), dict(num_draft_layers=0),
+    dict(d_model=100), dict(d_model=0), dict(num_kv_heads=0), dict(head_dim=96),
+    dict(n_sink=-1), dict(window=0), dict(rope_theta=-1.0), dict(rope_theta=float("inf")),
+])
+def test_append_rejects_bad_desc(spire, kw):
+    d = _adesc(spire, **kw)
+    assert spire.spire_feedback_append_workspace_bytes(d) == 0
+    good = 1 << 20
+    st = spire.spire_feedback_append(good, good, good, good, d, good, good, 1 << 30, 0)
+    want = spire._lib.SPIRE_ERR_UNSUPPORTED if "head_dim" in kw else spire._lib.SPIRE_ERR_INVALID_ARG
+    assert st == want
+
+
+def test_append_rejects_bad_args(spire):
+    d = _adesc(spire)
+    ws = spire.spire_feedback_append_workspace_bytes(d)
+    good = 1 << 20
+    E = spire._lib
+    # null pointers, misalignment, small workspace: all refused before any launch
+    for i in range(6):
+        args = [good] * 6
+        args[i] = 0
+        x, mw, wkv, pos, kv, w = args
+        assert spire.spire_feedback_append(x, mw, wkv, pos, d, kv, w, ws, 0) == E.SPIRE_ERR_INVALID_ARG
+    assert spire.spire_feedback_append(good + 8, good, good, good, d, good, good, ws, 0) == \
+        E.SPIRE_ERR_INVALID_ARG
+    assert spire.spire_feedback_append(good, good, good, good, d, good, good + 16, ws, 0) == \
+        E.SPIRE_ERR_INVALID_ARG
+    assert spire.spire_feedback_append(good, good, good, good, d, good, good, ws - 1, 0) == \
+        E.SPIRE_ERR_WORKSPACE
+    assert spire.spire_feedback_append(good, good, good, good, None, good, good, ws, 0) == \
+        E.SPIRE_ERR_INVALID_ARG

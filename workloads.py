@@ -214,6 +214,40 @@ def make_draft(ctx_lens, num_q_heads: int, num_kv_heads: int, head_dim: int,
                        n_sink=n_sink, window=window)
 
 
+@dataclasses.dataclass
+class AppendInputs:
+    x: torch.Tensor           # bf16 [n_act, B, d_model]: the token's activations
+    mix_w: torch.Tensor       # fp32 [n_dl, n_act]: mixing weights (un-normalised)
+    w_kv: torch.Tensor        # bf16 [n_dl, 2*Hkv*D, d_model]: key rows, then value rows
+    pos: torch.Tensor         # int32 [B]: logical position of the new entry
+    kv: torch.Tensor          # bf16 [n_dl, B, 2, Hkv, n_sink + window, D]: caches
+    n_sink: int
+    window: int
+
+
+def make_append(pos, num_act: int, num_draft_layers: int, d_model: int, num_kv_heads: int,
+                head_dim: int, n_sink: int, window: int, *, seed: int,
+                device="cpu") -> AppendInputs:
+    """Inputs of the feedback-memory append: N(0,1) activations and mixing
+    weights, N(0, 1/d_model) projections (entries of order 1), caches filled
+    with N(0,1) bf16 so that untouched slots are recognisable."""
+    p = np.asarray(pos, dtype=np.int64)
+    B = int(p.size)
+    S = n_sink + window
+    gen = _gen(seed, device)
+    x = _randn_bf16((num_act, B, d_model), gen, device)
+    mix_w = torch.randn((num_draft_layers, num_act), generator=gen, device=device,
+                        dtype=torch.float32)
+    F = 2 * num_kv_heads * head_dim
+    w_kv = _randn_bf16((num_draft_layers, F, d_model), gen, device, 1.0 / math.sqrt(d_model))
+    kv = torch.empty((num_draft_layers, B, 2, num_kv_heads, S, head_dim), dtype=torch.bfloat16,
+                     device=device)
+    _randn_bf16_inplace(kv, gen)
+    return AppendInputs(x=x, mix_w=mix_w, w_kv=w_kv,
+                        pos=torch.from_numpy(p.astype(np.int32)).to(device), kv=kv,
+                        n_sink=n_sink, window=window)
+
+
 def bf16_bits(t: torch.Tensor) -> np.ndarray:
     """Raw bf16 bit patterns of a tensor as a host uint16 numpy array."""
     return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
