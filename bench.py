@@ -150,6 +150,14 @@ def draft_bytes(t, S, Hq, Hkv, D):
     return int(np.minimum(t, S).sum()) * 4 * Hkv * D + B * Hq * D * 6 + 4 * B
 
 
+def append_bytes(B, n_act, n_dl, d_model, Hkv, D):
+    """Algorithmic bytes of one feedback-memory append: the projection weights
+    once, the activations, the mixing weights, the new entries and positions."""
+    F = 2 * Hkv * D
+    return n_dl * F * d_model * 2 + n_act * B * d_model * 2 + n_dl * n_act * 4 + \
+        n_dl * B * F * 2 + 4 * B
+
+
 def verify_flops(L, k, Hq, D):
     L = np.asarray(L, dtype=np.int64)
     rows = sum(int((L - k + i).sum()) for i in range(k + 1))
@@ -410,6 +418,75 @@ def spire_arm(args, cfg):
         e2e_ms.append(a.elapsed_time(b))
     e2e_val = job_value(tokens, world, reduce_max([statistics.mean(e2e_ms)], dist, dev)[0])
 
+    # ---- draft-step pipeline: a draft with n_dl = 2 layers (3 activations mixed,
+    # d_model = Hq * D); each step attends on every layer's cache, then appends
+    # the new feedback-memory entry to every cache (spire_feedback_append)
+    n_dl, n_act, d_model = 2, 3, Hq * D
+    t0s = wl.draft_ctx_for_step(L, k, 0)
+    ai = wl.make_append(t0s, n_act, n_dl, d_model, Hkv, D, cfg.n_sink, cfg.window,
+                        seed=cfg.seed + 101, device=dev)
+    adesc = spire.make_append_desc(B, n_act, n_dl, d_model, Hkv, D, cfg.n_sink, cfg.window,
+                                   10000.0)
+    ws_a = torch.empty(spire.spire_feedback_append_workspace_bytes(adesc), dtype=torch.uint8,
+                       device=dev)
+    out_l = [torch.empty(d.q.shape, dtype=torch.float32, device=dev) for d in drafts]
+
+    def call_append(j, s_handle=None):
+        st = spire.spire_feedback_append(ai.x, ai.mix_w, ai.w_kv, drafts[j].ctx_lens, adesc,
+                                         ai.kv, ws_a, ws_a.numel(), s_handle or sptr)
+        if st:
+            raise spire.SpireError(st, "spire_feedback_append")
+
+    def draft_round(s_handle=None):
+        for j in range(k):
+            for li in range(n_dl):
+                st = spire.spire_draft_sparse_attention(
+                    drafts[j].q, ai.kv[li], drafts[j].ctx_lens, cfg.n_sink, cfg.window, ddesc,
+                    out_l[j], ws_d, ws_d.numel(), s_handle or sptr)
+                if st:
+                    raise spire.SpireError(st, "spire_draft_sparse_attention")
+            call_append(j, s_handle)
+
+    for _ in range(max(3, args.warmup)):
+        call_append(0)
+    torch.cuda.synchronize(dev)
+    if spire.spire_get_device_error(ws_a, stream):
+        raise RuntimeError("device error word set by spire_feedback_append")
+    a_steps = max(1, min(args.steps, 200))
+    a_ev = []
+    for s in range(a_steps):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call_append(s % k)
+        b.record(stream)
+        a_ev.append((a, b))
+    torch.cuda.synchronize(dev)
+    app_ms = statistics.mean(a.elapsed_time(b) for a, b in a_ev)
+    pgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cap):
+        draft_round(cap.cuda_stream)
+        torch.cuda.synchronize(dev)
+        with torch.cuda.graph(pgraph, stream=cap):
+            draft_round(cap.cuda_stream)
+    stream.wait_stream(cap)
+    for _ in range(max(3, args.warmup)):
+        pgraph.replay()
+    torch.cuda.synchronize(dev)
+    p_ev = []
+    for s in range(a_steps):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        pgraph.replay()
+        b.record(stream)
+        p_ev.append((a, b))
+    torch.cuda.synchronize(dev)
+    pipe_ms = statistics.mean(a.elapsed_time(b) for a, b in p_ev)
+    del pgraph
+    app_ms, pipe_ms = reduce_max([app_ms, pipe_ms], dist, dev)
+    ab = append_bytes(B, n_act, n_dl, d_model, Hkv, D)
+
     if rank != 0:
         if dist is not None:
             dist.barrier()
@@ -453,7 +530,19 @@ def spire_arm(args, cfg):
                    "verify_tokens_per_s": world * tokens / (v_ms * 1e-3),
                    "draft_tokens_per_s": world * B * k / (d_ms * 1e-3),
                    "verify_tflops": verify_flops(L, k, Hq, D) / (v_ms * 1e-3) / 1e12,
-                   "tau_weighted_tokens_per_s_context": world * B * SPIRE_TAU_K4_L512 / (ms * 1e-3)},
+                   "tau_weighted_tokens_per_s_context": world * B * SPIRE_TAU_K4_L512 / (ms * 1e-3),
+                   "feedback_append": {
+                       "shape": "%d draft layers, %d activations, d_model %d, %d KV heads x %d, "
+                                "keys rotated (theta 1e4)" % (n_dl, n_act, d_model, Hkv, D),
+                       "us": app_ms * 1e3, "algorithmic_bytes": ab,
+                       "gbs": ab / (app_ms * 1e-3) / 1e9,
+                       "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
+                       "launches": 3},
+                   "draft_step_pipeline": {
+                       "what": "one CUDA graph per round: %d steps x (%d layer attention calls + "
+                               "one feedback append)" % (k, n_dl),
+                       "ms_per_round": pipe_ms,
+                       "draft_tokens_per_s": world * B * k / (pipe_ms * 1e-3)}},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h)},

@@ -225,7 +225,8 @@ typedef struct spire_append_desc {
 
 /*
  * spire_feedback_append_workspace_bytes -- workspace size for
- * spire_feedback_append (split-K partials and the device error word).
+ * spire_feedback_append (the memory vectors as two bf16 parts, split-K
+ * partials, rotary frequencies and the device error word).
  * Returns 0 for invalid arguments.
  */
 SPIRE_API size_t spire_feedback_append_workspace_bytes(const spire_append_desc *desc);
