@@ -181,6 +181,28 @@ def job_value(tokens_per_rank, world, step_ms):
     return world * tokens_per_rank / (step_ms * 1e-3)
 
 
+def perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms):
+    """Attention-only iteration time multiplier of one layer (Section 2) from
+    the measured kernels, beside the model's memory-bound prediction from the
+    algorithmic bytes (HOI cancels when every pass is memory-bound)."""
+    from paper_2504_06419_gb300 import perf_model as pm
+    L = np.asarray(L, dtype=np.int64)
+    t_draft = d_ms / k
+    dt = pm.measured_delta_t(k, t_draft, v_ms, dec_ms)
+    db = sum(draft_bytes(wl.draft_ctx_for_step(L, k, j), S, Hq, Hkv, D) for j in range(k)) / k
+    # one attention layer has no weights, and its FLOPs are far below bytes x HOI
+    # here, so each pass costs its KV bytes (the paper's form: the target pass and
+    # the verification read the same KV_target)
+    modeled = pm.iteration_time_multiplier(k, 0.0, 0.0, db, 0.0, 0.0,
+                                           verify_bytes(L, k, Hq, Hkv, D), 1.0)
+    return {"what": "one attention layer: delta_t = (k t_draft + t_verify) / t_decode, t_decode = "
+                    "the verify kernel with k = 0 at length L - k",
+            "t_decode_ms": dec_ms, "t_verify_ms": v_ms, "t_draft_ms": t_draft,
+            "delta_t_measured": dt, "delta_t_memory_bound_model": modeled,
+            "tau_context": SPIRE_TAU_K4_L512,
+            "throughput_multiplier_context": pm.throughput_multiplier(SPIRE_TAU_K4_L512, dt)}
+
+
 # ------------------------------------------------------------------ oracle arm
 def run_oracle_sample(cfg, n_seq, threads):
     """Time the fp64 oracle on the first n_seq sequences of the workload:
@@ -332,6 +354,31 @@ def spire_arm(args, cfg):
     v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
     d_ms = statistics.mean(sum(e[1 + j].elapsed_time(e[2 + j]) for j in range(k)) for e in ev)
 
+    # ---- plain decoding on the same cache (verify with k = 0 at length L - k): t_target
+    q0 = vi.q[:, :1].contiguous()
+    ctx0 = (vi.ctx_lens - k).contiguous()
+    out0 = torch.empty(q0.shape, dtype=torch.float32, device=dev)
+    ws0 = torch.empty(spire.spire_verify_workspace_bytes(vdesc, 0), dtype=torch.uint8, device=dev)
+
+    def call_decode():
+        st = spire.spire_verify_attention(q0, vi.k_cache, vi.v_cache, vi.block_table, ctx0, 0,
+                                          vdesc, out0, ws0, ws0.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_verify_attention (k = 0)")
+
+    for _ in range(args.warmup):
+        call_decode()
+    dec_ev = []
+    for s in range(n_detail):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call_decode()
+        b.record(stream)
+        dec_ev.append((a, b))
+    barrier()
+    dec_ms = statistics.mean(a.elapsed_time(b) for a, b in dec_ev)
+
     # ---- the round as one CUDA graph (verify + k draft steps), replayed per step
     graph = torch.cuda.CUDAGraph()
     cap = torch.cuda.Stream(dev)
@@ -365,7 +412,7 @@ def spire_arm(args, cfg):
     t1 = time.time()
     clocks = sampler.stop(t0, t1)
     ms = statistics.mean(e[0].elapsed_time(e[1]) for e in gev)
-    ms, eager_ms, v_ms, d_ms = reduce_max([ms, eager_ms, v_ms, d_ms], dist, dev)
+    ms, eager_ms, v_ms, d_ms, dec_ms = reduce_max([ms, eager_ms, v_ms, d_ms, dec_ms], dist, dev)
     del graph
 
     B = int(L.size)
@@ -538,6 +585,7 @@ def spire_arm(args, cfg):
                        "gbs": ab / (app_ms * 1e-3) / 1e9,
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "launches": 3},
+                   "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
                    "draft_step_pipeline": {
                        "what": "one CUDA graph per round: %d steps x (%d layer attention calls + "
                                "one feedback append)" % (k, n_dl),

@@ -21,6 +21,7 @@ Functions (each follows the passage cited in ``spire_oracle.c``):
   feedback_mix(...)    per-layer feedback memory vectors (Section 3.3)
   feedback_append(...) memory vector -> K/V projection -> bounded-cache slot
   round_bf16(v)        nearest-even bf16 bits of a double
+  verify_tokens(...)   modified rejection sampling of a round's draft tokens
 """
 from __future__ import annotations
 
@@ -73,6 +74,8 @@ def _declare(lib):
     lib.oracle_round_bf16.argtypes = [_F64]
     lib.oracle_feedback_mix.restype = _I64
     lib.oracle_feedback_mix.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _P]
+    lib.oracle_verify_tokens.restype = _I64
+    lib.oracle_verify_tokens.argtypes = [_P, _P, _P, _P, _P, _I32, _I32, _I32, _P, _P]
     lib.oracle_feedback_append.restype = _I64
     lib.oracle_feedback_append.argtypes = [_P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32,
                                            _I32, _I32, _F64, _P]
@@ -248,3 +251,27 @@ def feedback_append(x, w, w_kv, pos, kv, n_sink, window, rope_theta=0.0, lib=Non
     if n_bad < 0:
         raise ValueError("oracle_feedback_append rejected its arguments")
     return int(n_bad)
+
+
+def verify_tokens(p, q, x, u, e, lib=None):
+    """Token verification of one round per sequence.
+
+    p float32 [B, k+1, V], q float32 [B, k, V], x int32 [B, k], u float32 [B, k],
+    e float32 [B, V].  Returns (out int32 [B, k+1], n_accepted int32 [B], n_bad)."""
+    lib = lib or load()
+    p = np.ascontiguousarray(p, dtype=np.float32)
+    q = np.ascontiguousarray(q, dtype=np.float32)
+    x = _i32(x)
+    u = np.ascontiguousarray(u, dtype=np.float32)
+    e = np.ascontiguousarray(e, dtype=np.float32)
+    B, kp1, V = p.shape
+    k = kp1 - 1
+    if q.shape != (B, k, V) or x.shape != (B, k) or u.shape != (B, k) or e.shape != (B, V):
+        raise ValueError("verify_tokens: shape mismatch")
+    out = np.zeros((B, kp1), dtype=np.int32)
+    n_acc = np.zeros(B, dtype=np.int32)
+    n_bad = lib.oracle_verify_tokens(_ptr(p), _ptr(q), _ptr(x), _ptr(u), _ptr(e), B, k, V,
+                                     _ptr(out), _ptr(n_acc))
+    if n_bad < 0:
+        raise ValueError("oracle_verify_tokens rejected its arguments")
+    return out, n_acc, int(n_bad)

@@ -30,6 +30,10 @@
  *                         equation and the per-layer memory equation).
  *   oracle_draft_slot  -- where logical memory position p lives in the
  *                         bounded cache (sinks fixed, window a ring).
+ *   oracle_feedback_*  -- the draft step's memory vector and its K/V entry in
+ *                         the bounded cache (Section 3.3).
+ *   oracle_verify_tokens -- modified rejection sampling of a round's draft
+ *                         tokens (Section 1; Section 6).
  *
  * Readings of points the paper leaves open (all listed in the design doc):
  *   - scores are softmax_scale * <q, k>; the workloads pre-scale q, scale = 1;
@@ -576,5 +580,117 @@ int64_t oracle_feedback_append(const uint16_t *x, const double *w,
     }
     free(m);
     free(y);
+    return n_bad;
+}
+
+/* ======================================================================== */
+/* Token verification (modified rejection sampling)                          */
+/* ======================================================================== */
+/*
+ * The target accepts the draft tokens of a round one by one so that every
+ * emitted token is a sample of the target's own distribution (Section 1:
+ * modified rejection sampling; the token verification algorithm of the
+ * paper's experiments, Section 6).  For sequence b with drafts x_1..x_k drawn
+ * from the draft distributions q_1..q_k and target distributions p_1..p_{k+1}
+ * from the verification pass:
+ *   - draft i is accepted with probability min(1, p_i(x_i) / q_i(x_i)): with a
+ *     uniform u_i in [0, 1), accepted iff u_i * q_i(x_i) < p_i(x_i);
+ *   - at the first rejected i the round emits a token drawn from
+ *     norm(max(0, p_i - q_i)) and stops; if all k are accepted it emits a
+ *     bonus token drawn from p_{k+1}.
+ * Readings: a draw from weights w is the exponential race
+ * argmax_v w_v / E_v over w_v > 0 with E_v ~ Exp(1) given as input (ties to
+ * the smallest v), which selects v with probability w_v / sum w; every
+ * comparison, product, difference and quotient is taken in binary32, as the
+ * kernel does, so both sides take the same integer decisions; if the
+ * residual has no positive entry the draw uses p_i itself; a draft token
+ * outside [0, V) counts as rejected, an E_v that is not > 0 is skipped, and
+ * both are reported.
+ */
+static uint64_t race_key(float w, float e, int32_t v)
+{
+    /* larger key = better candidate: the score's bits (scores are >= 0, so
+     * their bit patterns order like the values), then the smaller index */
+    float s = w / e;
+    uint32_t sb;
+    memcpy(&sb, &s, sizeof(sb));
+    return ((uint64_t)sb << 32) | (uint64_t)(~(uint32_t)v);
+}
+
+/* argmax_v w_v / e_v over w_v > 0, e_v > 0; returns -1 if no candidate. */
+static int32_t race_draw(const float *p, const float *q, int use_residual,
+                         const float *e, int32_t V, int32_t *bad_e)
+{
+    uint64_t best = 0;
+    int32_t arg = -1;
+    for (int32_t v = 0; v < V; ++v) {
+        if (!(e[v] > 0.0f)) {
+            *bad_e = 1;
+            continue;
+        }
+        float w = use_residual ? p[v] - q[v] : p[v];
+        if (!(w > 0.0f))
+            continue;
+        uint64_t key = race_key(w, e[v], v);
+        if (key > best) {
+            best = key;
+            arg = v;
+        }
+    }
+    return arg;
+}
+
+/*
+ * oracle_verify_tokens:
+ *   p       float [B, k+1, V]   target distributions p_1..p_{k+1}
+ *   q       float [B, k, V]     draft distributions q_1..q_k
+ *   x       int32 [B, k]        draft tokens x_1..x_k
+ *   u       float [B, k]        acceptance uniforms
+ *   e       float [B, V]        Exp(1) variates for the round's one draw
+ *   out     int32 [B, k+1]      x_1..x_j, then the drawn token, then -1
+ *   n_acc   int32 [B]           j, the number of accepted drafts
+ * Returns the number of sequences with an invalid draft token, E value or an
+ * empty distribution (their draw may be -1), or -1 on bad arguments.
+ */
+int64_t oracle_verify_tokens(const float *p, const float *q, const int32_t *x,
+                             const float *u, const float *e, int32_t B,
+                             int32_t k, int32_t V, int32_t *out,
+                             int32_t *n_acc)
+{
+    if (B < 0 || k < 0 || V < 1)
+        return -1;
+    int64_t n_bad = 0;
+    for (int32_t b = 0; b < B; ++b) {
+        int32_t bad = 0;
+        int32_t j = 0;
+        for (; j < k; ++j) {
+            int32_t t = x[(int64_t)b * k + j];
+            if (t < 0 || t >= V) {
+                bad = 1;
+                break;
+            }
+            float pv = p[((int64_t)b * (k + 1) + j) * V + t];
+            float qv = q[((int64_t)b * k + j) * V + t];
+            float uq = u[(int64_t)b * k + j] * qv;
+            if (!(uq < pv))
+                break;
+        }
+        const float *pj = p + ((int64_t)b * (k + 1) + j) * V;
+        const float *qj = j < k ? q + ((int64_t)b * k + j) * V : NULL;
+        const float *eb = e + (int64_t)b * V;
+        int32_t y = race_draw(pj, qj, j < k, eb, V, &bad);
+        if (y < 0 && j < k)
+            y = race_draw(pj, qj, 0, eb, V, &bad);
+        if (y < 0)
+            bad = 1;
+        int32_t *o = out + (int64_t)b * (k + 1);
+        for (int32_t i = 0; i < j; ++i)
+            o[i] = x[(int64_t)b * k + i];
+        o[j] = y;
+        for (int32_t i = j + 1; i <= k; ++i)
+            o[i] = -1;
+        n_acc[b] = j;
+        n_bad += bad;
+    }
     return n_bad;
 }

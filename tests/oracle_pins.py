@@ -547,4 +547,110 @@ def pin_feedback_append_negative_position(lib):
     assert not np.array_equal(kv[:, 1], kv0[:, 1])
 
 
+# --------------------------------------------------------------------------
+# token verification (modified rejection sampling) pins
+# --------------------------------------------------------------------------
+def pin_tokens_hand_example(lib):
+    """Two sequences worked by hand (V = 4, k = 2).
+    Sequence 0: draft 3 is accepted (0.9 * 0.25 < 0.4), draft 1 rejected
+    (0.5 * 0.6 >= 0.1); residual max(0, p2 - q2) = (0.4, 0, 0, 0.2) with
+    E = (1, .5, .5, .3) scores 0.4 and 0.667: token 3.  Sequence 1: both drafts
+    accepted; bonus from p3 = (0, .7, .3, 0) with E = (1, 2, .25, 1): scores
+    0.35 and 1.2, token 2."""
+    p = np.array([[[0.1, 0.2, 0.3, 0.4], [0.5, 0.1, 0.1, 0.3], [0.0, 0.7, 0.3, 0.0]],
+                  [[0.1, 0.2, 0.3, 0.4], [0.5, 0.1, 0.1, 0.3], [0.0, 0.7, 0.3, 0.0]]],
+                 dtype=np.float32)
+    q = np.array([[[0.25, 0.25, 0.25, 0.25], [0.1, 0.6, 0.2, 0.1]],
+                  [[0.25, 0.25, 0.25, 0.25], [0.4, 0.1, 0.4, 0.1]]], dtype=np.float32)
+    x = np.array([[3, 1], [2, 0]], dtype=np.int32)
+    u = np.array([[0.9, 0.5], [0.5, 0.9]], dtype=np.float32)
+    e = np.array([[1.0, 0.5, 0.5, 0.3], [1.0, 2.0, 0.25, 1.0]], dtype=np.float32)
+    out, n_acc, n_bad = oracle.verify_tokens(p, q, x, u, e, lib=lib)
+    assert n_bad == 0
+    assert out.tolist() == [[3, 3, -1], [2, 0, 2]] and n_acc.tolist() == [1, 2]
+
+
+def _round_samples(rng, n, p_rows, q_rows):
+    """n independent rounds with fixed distributions: drafts drawn from q_i,
+    uniforms and Exp(1) variates from numpy."""
+    kp1, V = p_rows.shape
+    k = kp1 - 1
+    qd = q_rows.astype(np.float64)
+    x = np.stack([rng.choice(V, size=n, p=qd[i] / qd[i].sum()) for i in range(k)],
+                 axis=1).astype(np.int32)
+    u = rng.random((n, k), dtype=np.float32)
+    e = rng.exponential(size=(n, V)).astype(np.float32)
+    p = np.broadcast_to(p_rows, (n, kp1, V))
+    q = np.broadcast_to(q_rows, (n, k, V))
+    return p, q, x, u, e
+
+
+def _chi2_ok(counts, probs):
+    from scipy.stats import chisquare
+    keep = probs > 0
+    assert counts[~keep].sum() == 0, "a token of probability 0 was emitted"
+    return chisquare(counts[keep], counts[keep].sum() * probs[keep] / probs[keep].sum()).pvalue
+
+
+def pin_tokens_emitted_tokens_follow_the_target(lib):
+    """The scheme's guarantee (Section 1): the first emitted token is a sample
+    of p_1, and, where the first draft was accepted, the second of p_2 (the
+    synthetic distributions do not depend on the prefix)."""
+    rng = np.random.default_rng(41)
+    V, k, n = 6, 3, 120000
+    p_rows = rng.dirichlet(np.ones(V), size=k + 1).astype(np.float32)
+    q_rows = rng.dirichlet(np.ones(V), size=k).astype(np.float32)
+    p, q, x, u, e = _round_samples(rng, n, p_rows, q_rows)
+    out, n_acc, _ = oracle.verify_tokens(p, q, x, u, e, lib=lib)
+    c0 = np.bincount(out[:, 0], minlength=V)
+    assert _chi2_ok(c0, p_rows[0].astype(np.float64)) > 1e-4
+    sel = n_acc >= 1
+    c1 = np.bincount(out[sel, 1], minlength=V)
+    assert _chi2_ok(c1, p_rows[1].astype(np.float64)) > 1e-4
+
+
+def pin_tokens_acceptance_rate_is_alpha(lib):
+    """A draft drawn from q is accepted with probability
+    alpha = sum_v min(p_v, q_v), the expected acceptance probability
+    (Section 3.4)."""
+    rng = np.random.default_rng(42)
+    V, k, n = 8, 1, 200000
+    p_rows = rng.dirichlet(np.ones(V), size=k + 1).astype(np.float32)
+    q_rows = rng.dirichlet(np.ones(V), size=k).astype(np.float32)
+    p, q, x, u, e = _round_samples(rng, n, p_rows, q_rows)
+    _, n_acc, _ = oracle.verify_tokens(p, q, x, u, e, lib=lib)
+    alpha = np.minimum(p_rows[0].astype(np.float64), q_rows[0]).sum()
+    rate = (n_acc == 1).mean()
+    assert abs(rate - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / n)
+
+
+def pin_tokens_identical_models_accept_all(lib):
+    """p_i = q_i: every draft is accepted (u < 1) and the bonus token is a
+    sample of p_{k+1}."""
+    rng = np.random.default_rng(43)
+    V, k, n = 5, 2, 100000
+    rows = rng.dirichlet(np.ones(V), size=k + 1).astype(np.float32)
+    p, q, x, u, e = _round_samples(rng, n, rows, rows[:k])
+    out, n_acc, _ = oracle.verify_tokens(p, q, x, u, e, lib=lib)
+    assert np.all(n_acc == k) and np.array_equal(out[:, :k], x)
+    assert _chi2_ok(np.bincount(out[:, k], minlength=V), rows[k].astype(np.float64)) > 1e-4
+
+
+def pin_tokens_invalid_inputs(lib):
+    """A draft token outside [0, V) counts as rejected; an Exp value that is
+    not > 0 is skipped; both are counted."""
+    p = np.full((2, 2, 3), 1.0 / 3, dtype=np.float32)
+    q = np.full((2, 1, 3), 1.0 / 3, dtype=np.float32)
+    x = np.array([[7], [1]], dtype=np.int32)
+    u = np.zeros((2, 1), dtype=np.float32)
+    e = np.array([[1.0, 1.0, 1.0], [0.0, 2.0, 1.0]], dtype=np.float32)
+    out, n_acc, n_bad = oracle.verify_tokens(p, q, x, u, e, lib=lib)
+    assert n_bad == 2
+    assert n_acc.tolist() == [0, 1]
+    # sequence 0: residual of p = q is empty, so the draw falls back to p (ties: token 0)
+    assert out[0].tolist() == [0, -1]
+    # sequence 1: bonus from p_2 with E_0 skipped: scores (1/3)/2 and (1/3)/1 -> token 2
+    assert out[1].tolist() == [1, 2]
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -59,6 +59,16 @@ MUTATIONS = [
      "double r = ldexp(trunc(ldexp(v, -q)), q);"),
     ("round_ties_away", "double r = ldexp(nearbyint(ldexp(v, -q)), q);",
      "double r = ldexp(round(ldexp(v, -q)), q);"),
+    ("accept_ratio_inverted", "float uq = u[(int64_t)b * k + j] * qv;",
+     "float uq = u[(int64_t)b * k + j] * pv; pv = qv;"),
+    ("residual_sign", "float w = use_residual ? p[v] - q[v] : p[v];",
+     "float w = use_residual ? q[v] - p[v] : p[v];"),
+    ("bonus_from_last_draft_row", "const float *pj = p + ((int64_t)b * (k + 1) + j) * V;",
+     "const float *pj = p + ((int64_t)b * (k + 1) + (j < k ? j : k - 1)) * V;"),
+    ("race_multiplies", "float s = w / e;", "float s = w * e;"),
+    ("race_argmin", "if (key > best) {", "if (best == 0 || key < best) {"),
+    ("accepted_tokens_reversed", "o[i] = x[(int64_t)b * k + i];",
+     "o[i] = x[(int64_t)b * k + (j - 1 - i)];"),
 ]
 
 
