@@ -158,6 +158,16 @@ def append_bytes(B, n_act, n_dl, d_model, Hkv, D):
         n_dl * B * F * 2 + 4 * B
 
 
+def tokens_bytes(n_acc, k, V):
+    """Algorithmic bytes of one token verification: per sequence the target row
+    of the draw and the Exp(1) row, the draft row when a draft was rejected,
+    the k gathered entries of p and q, the uniforms, tokens and outputs."""
+    n_acc = np.asarray(n_acc, dtype=np.int64)
+    B = n_acc.size
+    rows = B * 2 * V * 4 + int((n_acc < k).sum()) * V * 4
+    return rows + B * (k * 4 * 4 + (k + 1) * 4 + 4)
+
+
 def verify_flops(L, k, Hq, D):
     L = np.asarray(L, dtype=np.int64)
     rows = sum(int((L - k + i).sum()) for i in range(k + 1))
@@ -533,6 +543,39 @@ def spire_arm(args, cfg):
     del pgraph
     app_ms, pipe_ms = reduce_max([app_ms, pipe_ms], dist, dev)
     ab = append_bytes(B, n_act, n_dl, d_model, Hkv, D)
+    del ai, ws_a
+
+    # ---- token verification of the round (modified rejection sampling), a
+    # Llama 3 sized vocabulary as the stand-in (the paper extrapolates to it)
+    V_tok = 128256
+    ti = wl.make_tokens(B, k, V_tok, seed=cfg.seed + 202, device=dev)
+    ws_t = torch.empty(spire.spire_verify_tokens_workspace_bytes(B, k, V_tok), dtype=torch.uint8,
+                       device=dev)
+    tok_out = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+    tok_acc = torch.empty((B,), dtype=torch.int32, device=dev)
+
+    def call_tokens():
+        st = spire.spire_verify_tokens(ti.p, ti.q, ti.x, ti.u, ti.e, B, k, V_tok, tok_out,
+                                       tok_acc, ws_t, ws_t.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_verify_tokens")
+
+    for _ in range(max(3, args.warmup)):
+        call_tokens()
+    torch.cuda.synchronize(dev)
+    t_ev = []
+    for s in range(a_steps):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call_tokens()
+        b.record(stream)
+        t_ev.append((a, b))
+    torch.cuda.synchronize(dev)
+    tok_ms = reduce_max([statistics.mean(a.elapsed_time(b) for a, b in t_ev)], dist, dev)[0]
+    n_acc_h = tok_acc.cpu().numpy()
+    tb = tokens_bytes(n_acc_h, k, V_tok)
+    del ti
 
     if rank != 0:
         if dist is not None:
@@ -586,6 +629,12 @@ def spire_arm(args, cfg):
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "launches": 3},
                    "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
+                   "verify_tokens": {
+                       "shape": "B=%d, k=%d, vocabulary %d (fp32 distributions)" % (B, k, V_tok),
+                       "us": tok_ms * 1e3, "algorithmic_bytes": tb,
+                       "gbs": tb / (tok_ms * 1e-3) / 1e9,
+                       "frac": tb / (tok_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
+                       "mean_accepted": float(n_acc_h.mean()), "launches": 2},
                    "draft_step_pipeline": {
                        "what": "one CUDA graph per round: %d steps x (%d layer attention calls + "
                                "one feedback append)" % (k, n_dl),

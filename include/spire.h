@@ -21,6 +21,9 @@
  *                                 token's activations into each layer's memory
  *                                 vector, project it to K/V and store it in
  *                                 the bounded cache (Section 3.3).
+ *   spire_verify_tokens           the round's token verification: modified
+ *                                 rejection sampling of the draft tokens
+ *                                 (Section 1).
  *
  * Conventions common to every call
  *   - All tensor arguments are DEVICE pointers, owned by the caller; the
@@ -70,6 +73,7 @@ typedef enum spire_status {
 #define SPIRE_DEVERR_CTX_LEN 1u  /* a ctx_lens entry outside its allowed range */
 #define SPIRE_DEVERR_PAGE_ID 2u  /* a block_table entry outside [0, num_pages) */
 #define SPIRE_DEVERR_TIMEOUT 4u  /* a bounded wait inside a kernel gave up */
+#define SPIRE_DEVERR_VALUE 8u    /* an input value outside its domain (spire_verify_tokens) */
 
 /* Shapes shared by both kernels. */
 typedef struct spire_attn_desc {
@@ -260,6 +264,57 @@ SPIRE_API spire_status spire_feedback_append(const void *x, const float *mix_w,
                                              const spire_append_desc *desc, void *kv,
                                              void *workspace, size_t ws_bytes,
                                              void *stream);
+
+/*
+ * Token verification of a speculation round (modified rejection sampling).
+ *
+ * Every emitted token is a sample of the target's own distribution (Section
+ * 1; the token verification algorithm of the paper's experiments, Section 6).
+ * For sequence b with draft tokens x_1..x_k drawn from the draft
+ * distributions q_1..q_k and target distributions p_1..p_{k+1} from the
+ * verification pass:
+ *   - draft i is accepted with probability min(1, p_i(x_i) / q_i(x_i)): with a
+ *     uniform u_i in [0, 1), accepted iff u_i * q_i(x_i) < p_i(x_i) (binary32);
+ *     j is the number of leading accepted drafts;
+ *   - the round then draws one token: from max(0, p_{j+1} - q_{j+1})
+ *     normalised when j < k (from p_{j+1} if that residual has no positive
+ *     entry), from p_{k+1} when j = k.  A draw from weights w is the
+ *     exponential race argmax_v w_v / E_v over w_v > 0 (binary32 quotient, ties
+ *     to the smallest v) with E_v ~ Exp(1) supplied by the caller, which picks
+ *     v with probability w_v / sum(w).
+ * Random numbers are inputs, so a call is deterministic.
+ */
+
+/*
+ * spire_verify_tokens_workspace_bytes -- workspace size for
+ * spire_verify_tokens (one partial per sequence and 8192-entry vocabulary
+ * chunk, and the device error word).  Returns 0 for invalid shapes.
+ */
+SPIRE_API size_t spire_verify_tokens_workspace_bytes(int32_t batch, int32_t k, int32_t vocab);
+
+/*
+ * spire_verify_tokens --
+ *   p            fp32 [B, k+1, V]: target distributions p_1..p_{k+1}.
+ *   q            fp32 [B, k, V]:   draft distributions q_1..q_k (may be NULL if k = 0).
+ *   draft_tokens int32 [B, k]:     x_1..x_k (may be NULL if k = 0).
+ *   u            fp32 [B, k]:      acceptance uniforms in [0, 1) (may be NULL if k = 0).
+ *   e            fp32 [B, V]:      Exp(1) variates for the round's one draw.
+ *   batch 1..65535, k 0..31, vocab V >= 1.
+ *   out_tokens   int32 [B, k+1]:   x_1..x_j, the drawn token, then -1.
+ *   n_accepted   int32 [B]:        j.
+ * Only the rows the round needs are read (p_{j+1}, q_{j+1}, E and k gathered
+ * entries).  A draft token outside [0, V) counts as rejected and sets
+ * SPIRE_DEVERR_CTX_LEN; an E value that is not > 0 is skipped, and a draw with
+ * no candidate yields -1; both set SPIRE_DEVERR_VALUE.  Pointers must be
+ * 4-byte aligned (p, q and e 16-byte aligned when V is a multiple of 4), the
+ * workspace 256-byte aligned.
+ */
+SPIRE_API spire_status spire_verify_tokens(const float *p, const float *q,
+                                           const int32_t *draft_tokens, const float *u,
+                                           const float *e, int32_t batch, int32_t k,
+                                           int32_t vocab, int32_t *out_tokens,
+                                           int32_t *n_accepted, void *workspace,
+                                           size_t ws_bytes, void *stream);
 
 /*
  * spire_draft_slot -- slot of logical memory position p >= 0 in the bounded

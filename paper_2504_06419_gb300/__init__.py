@@ -13,6 +13,8 @@ libspire (include/spire.h):
   spire_feedback_append          the draft step's cache update: per-layer
                                  memory vector, K/V projection, bounded-cache
                                  slot (Section 3.3)
+  spire_verify_tokens            token verification: modified rejection
+                                 sampling of the round's drafts (Section 1)
 
 The functions below allocate outputs and workspaces with PyTorch and call the
 C ABI; all computation runs in the library's kernels.
@@ -26,12 +28,14 @@ from ._lib import (SpireError, make_append_desc, make_desc, spire_draft_slot,
                    spire_draft_sparse_attention, spire_draft_workspace_bytes,
                    spire_feedback_append, spire_feedback_append_workspace_bytes,
                    spire_get_device_error, spire_status_string, spire_verify_attention,
-                   spire_verify_attention_noalloc, spire_verify_workspace_bytes)
+                   spire_verify_attention_noalloc, spire_verify_tokens,
+                   spire_verify_tokens_workspace_bytes, spire_verify_workspace_bytes)
 
 __all__ = [
     "SpireError", "make_desc", "make_append_desc", "spire_verify_attention",
     "spire_verify_attention_noalloc", "spire_draft_sparse_attention", "spire_feedback_append",
-    "spire_feedback_append_workspace_bytes", "feedback_append",
+    "spire_feedback_append_workspace_bytes", "feedback_append", "spire_verify_tokens",
+    "spire_verify_tokens_workspace_bytes", "verify_tokens",
     "spire_verify_workspace_bytes", "spire_draft_workspace_bytes", "spire_draft_slot",
     "spire_get_device_error", "spire_status_string", "verify_attention", "draft_attention",
     "verify_desc", "draft_desc",
@@ -101,3 +105,25 @@ def feedback_append(x, mix_w, w_kv, pos, kv, n_sink, window, rope_theta=0.0, wor
     if st != 0:
         raise SpireError(st, "spire_feedback_append")
     return kv
+
+
+def verify_tokens(p, q, draft_tokens, u, e, workspace=None, stream=None):
+    """Token verification of one round per sequence (modified rejection
+    sampling).  p fp32 [B, k+1, V], q fp32 [B, k, V], draft_tokens int32 [B, k],
+    u fp32 [B, k], e fp32 [B, V] (Exp(1) variates), all on the GPU.
+    Returns (out_tokens int32 [B, k+1], n_accepted int32 [B])."""
+    B, kp1, V = p.shape
+    k = kp1 - 1
+    ws_bytes = spire_verify_tokens_workspace_bytes(B, k, V)
+    if ws_bytes == 0:
+        raise SpireError(1, "spire_verify_tokens_workspace_bytes")
+    if workspace is None:
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=p.device)
+    out = torch.empty((B, kp1), dtype=torch.int32, device=p.device)
+    n_acc = torch.empty((B,), dtype=torch.int32, device=p.device)
+    st = spire_verify_tokens(p, q if k > 0 else None, draft_tokens if k > 0 else None,
+                             u if k > 0 else None, e, B, k, V, out, n_acc, workspace,
+                             workspace.numel(), stream)
+    if st != 0:
+        raise SpireError(st, "spire_verify_tokens")
+    return out, n_acc

@@ -25,6 +25,7 @@ SPIRE_ERR_CUDA = 4
 SPIRE_DEVERR_CTX_LEN = 1
 SPIRE_DEVERR_PAGE_ID = 2
 SPIRE_DEVERR_TIMEOUT = 4
+SPIRE_DEVERR_VALUE = 8
 
 SPIRE_MAX_ROWS_PER_KV_HEAD = 128
 
@@ -36,6 +37,8 @@ EXPORTED = (
     "spire_draft_sparse_attention",
     "spire_feedback_append_workspace_bytes",
     "spire_feedback_append",
+    "spire_verify_tokens_workspace_bytes",
+    "spire_verify_tokens",
     "spire_draft_slot",
     "spire_get_device_error",
     "spire_status_string",
@@ -97,6 +100,10 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_feedback_append_workspace_bytes.argtypes = [A]
     lib.spire_feedback_append.restype = ctypes.c_int
     lib.spire_feedback_append.argtypes = [P, P, P, P, A, P, P, SZ, P]
+    lib.spire_verify_tokens_workspace_bytes.restype = SZ
+    lib.spire_verify_tokens_workspace_bytes.argtypes = [I32, I32, I32]
+    lib.spire_verify_tokens.restype = ctypes.c_int
+    lib.spire_verify_tokens.argtypes = [P, P, P, P, P, I32, I32, I32, P, P, P, SZ, P]
     lib.spire_draft_slot.restype = I64
     lib.spire_draft_slot.argtypes = [I64, I32, I32]
     lib.spire_get_device_error.restype = ctypes.c_int
@@ -186,6 +193,17 @@ def spire_feedback_append(x, mix_w, w_kv, pos, desc, kv, workspace, ws_bytes, st
     return int(LIB.spire_feedback_append(
         _ptr(x), _ptr(mix_w), _ptr(w_kv), _ptr(pos), _desc_ref(desc), _ptr(kv), _ptr(workspace),
         int(ws_bytes), _stream(stream, x)))
+
+
+def spire_verify_tokens_workspace_bytes(batch: int, k: int, vocab: int) -> int:
+    return int(LIB.spire_verify_tokens_workspace_bytes(int(batch), int(k), int(vocab)))
+
+
+def spire_verify_tokens(p, q, draft_tokens, u, e, batch, k, vocab, out_tokens, n_accepted,
+                        workspace, ws_bytes, stream=None) -> int:
+    return int(LIB.spire_verify_tokens(
+        _ptr(p), _ptr(q), _ptr(draft_tokens), _ptr(u), _ptr(e), int(batch), int(k), int(vocab),
+        _ptr(out_tokens), _ptr(n_accepted), _ptr(workspace), int(ws_bytes), _stream(stream, p)))
 
 
 def spire_draft_slot(pos: int, n_sink: int, window: int) -> int:

@@ -20,7 +20,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libspire.so")
-SOURCES = ["spire_abi.cu", "spire_split_d64.cu", "spire_split_d128.cu", "spire_append.cu"]
+SOURCES = ["spire_abi.cu", "spire_split_d64.cu", "spire_split_d128.cu", "spire_append.cu",
+           "spire_tokens.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -29,6 +29,7 @@ def test_header_declares_the_boundary():
         "spire_verify_workspace_bytes", "spire_verify_attention",
         "spire_verify_attention_noalloc", "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
         "spire_feedback_append_workspace_bytes", "spire_feedback_append",
+        "spire_verify_tokens_workspace_bytes", "spire_verify_tokens",
         "spire_get_device_error", "spire_status_string"]), names
 
 
@@ -177,3 +178,25 @@ def test_append_rejects_bad_args(spire):
         E.SPIRE_ERR_WORKSPACE
     assert spire.spire_feedback_append(good, good, good, good, None, good, good, ws, 0) == \
         E.SPIRE_ERR_INVALID_ARG
+
+
+def test_tokens_workspace_and_host_checks(spire):
+    E = spire._lib
+    assert spire.spire_verify_tokens_workspace_bytes(64, 4, 128256) == 512 + 64 * 16 * 24
+    assert spire.spire_verify_tokens_workspace_bytes(1, 0, 1) == 512 + 24
+    for bad in [(0, 4, 100), (1, -1, 100), (1, 32, 100), (1, 4, 0), (70000, 1, 10)]:
+        assert spire.spire_verify_tokens_workspace_bytes(*bad) == 0
+    good = 1 << 20
+    ws = spire.spire_verify_tokens_workspace_bytes(8, 4, 1000)
+    call = lambda **kw: spire.spire_verify_tokens(**{**dict(
+        p=good, q=good, draft_tokens=good, u=good, e=good, batch=8, k=4, vocab=1000,
+        out_tokens=good, n_accepted=good, workspace=good, ws_bytes=ws, stream=0), **kw})
+    for name in ("p", "q", "draft_tokens", "u", "e", "out_tokens", "n_accepted", "workspace"):
+        assert call(**{name: 0}) == E.SPIRE_ERR_INVALID_ARG, name
+    # with k = 0 the draft arguments may be NULL: refused only for the small workspace
+    assert call(k=0, q=0, draft_tokens=0, u=0, ws_bytes=0) == E.SPIRE_ERR_WORKSPACE
+    assert call(p=good + 4) == E.SPIRE_ERR_INVALID_ARG           # V % 4 == 0 needs 16 B
+    assert call(p=good + 2, vocab=1001) == E.SPIRE_ERR_INVALID_ARG
+    assert call(ws_bytes=ws - 1) == E.SPIRE_ERR_WORKSPACE
+    assert call(k=40) == E.SPIRE_ERR_UNSUPPORTED
+    assert call(batch=0) == E.SPIRE_ERR_INVALID_ARG

@@ -248,6 +248,37 @@ def make_append(pos, num_act: int, num_draft_layers: int, d_model: int, num_kv_h
                         n_sink=n_sink, window=window)
 
 
+@dataclasses.dataclass
+class TokenInputs:
+    p: torch.Tensor       # fp32 [B, k+1, V]: target distributions
+    q: torch.Tensor       # fp32 [B, k, V]: draft distributions
+    x: torch.Tensor       # int32 [B, k]: draft tokens, x_i drawn from q_i
+    u: torch.Tensor       # fp32 [B, k]: uniforms in [0, 1)
+    e: torch.Tensor       # fp32 [B, V]: Exp(1) variates
+
+
+def make_tokens(batch: int, k: int, vocab: int, *, seed: int, device="cpu",
+                logit_std: float = 2.0, draft_noise: float = 1.0) -> TokenInputs:
+    """Distributions of one speculation round: target logits N(0, logit_std^2)
+    per vocabulary entry, draft logits = target logits + N(0, draft_noise^2)
+    (a draft that roughly agrees with the target), both through a softmax;
+    draft tokens drawn from the draft distributions; uniforms and Exp(1)
+    variates from the same seeded generator."""
+    gen = _gen(seed, device)
+    zt = torch.randn((batch, k + 1, vocab), generator=gen, device=device) * logit_std
+    zd = zt[:, :k] + torch.randn((batch, k, vocab), generator=gen, device=device) * draft_noise
+    p = torch.softmax(zt, dim=-1).float().contiguous()
+    q = torch.softmax(zd, dim=-1).float().contiguous()
+    if k > 0:
+        x = torch.multinomial(q.reshape(batch * k, vocab), 1, generator=gen).reshape(batch, k)
+    else:
+        x = torch.zeros((batch, 0), dtype=torch.int64, device=device)
+    u = torch.rand((batch, k), generator=gen, device=device)
+    e = torch.empty((batch, vocab), device=device).exponential_(1.0, generator=gen)
+    return TokenInputs(p=p, q=q, x=x.to(torch.int32).contiguous(), u=u.contiguous(),
+                       e=e.contiguous())
+
+
 def bf16_bits(t: torch.Tensor) -> np.ndarray:
     """Raw bf16 bit patterns of a tensor as a host uint16 numpy array."""
     return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
