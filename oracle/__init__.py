@@ -22,6 +22,8 @@ Functions (each follows the passage cited in ``spire_oracle.c``):
   feedback_append(...) memory vector -> K/V projection -> bounded-cache slot
   round_bf16(v)        nearest-even bf16 bits of a double
   verify_tokens(...)   modified rejection sampling of a round's draft tokens
+  magicdec(...)        StreamingLLM draft attention over the target's paged cache
+                       with positions inside the reduced cache
 """
 from __future__ import annotations
 
@@ -74,6 +76,9 @@ def _declare(lib):
     lib.oracle_round_bf16.argtypes = [_F64]
     lib.oracle_feedback_mix.restype = _I64
     lib.oracle_feedback_mix.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _P]
+    lib.oracle_magicdec.restype = _I64
+    lib.oracle_magicdec.argtypes = [_P, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _I32,
+                                    _I32, _I32, _F64, _F64, _P]
     lib.oracle_verify_tokens.restype = _I64
     lib.oracle_verify_tokens.argtypes = [_P, _P, _P, _P, _P, _I32, _I32, _I32, _P, _P]
     lib.oracle_feedback_append.restype = _I64
@@ -275,3 +280,25 @@ def verify_tokens(p, q, x, u, e, lib=None):
     if n_bad < 0:
         raise ValueError("oracle_verify_tokens rejected its arguments")
     return out, n_acc, int(n_bad)
+
+
+def magicdec(q, k_cache, v_cache, block_table, ctx_lens, n_sink, window, rope_theta,
+             scale=1.0, lib=None):
+    """MagicDec draft attention: q bf16 bits [B, Hq, D] (not rotated), the
+    target's paged caches [num_pages, Hkv, page_size, D] (keys rotated by their
+    original positions), block_table [B, max_pages], ctx_lens [B].
+    Returns (out float64 [B, Hq, D], n_bad)."""
+    lib = lib or load()
+    q, kc, vc = _u16(q), _u16(k_cache), _u16(v_cache)
+    bt, cl = _i32(block_table), _i32(ctx_lens)
+    B, Hq, D = q.shape
+    num_pages, Hkv, page_size, D2 = kc.shape
+    if D2 != D or vc.shape != kc.shape:
+        raise ValueError("cache shape mismatch")
+    out = np.zeros((B, Hq, D), dtype=np.float64)
+    n_bad = lib.oracle_magicdec(_ptr(q), _ptr(kc), _ptr(vc), _ptr(bt), _ptr(cl), B, Hq, Hkv, D,
+                                page_size, bt.shape[1], num_pages, int(n_sink), int(window),
+                                float(rope_theta), float(scale), _ptr(out))
+    if n_bad < 0:
+        raise ValueError("oracle_magicdec rejected its arguments")
+    return out, int(n_bad)

@@ -34,6 +34,9 @@
  *                         the bounded cache (Section 3.3).
  *   oracle_verify_tokens -- modified rejection sampling of a round's draft
  *                         tokens (Section 1; Section 6).
+ *   oracle_magicdec    -- the MagicDec baseline's draft attention: sink +
+ *                         window over the target's own paged cache, positions
+ *                         inside the reduced cache (Section 3.1 footnote).
  *
  * Readings of points the paper leaves open (all listed in the design doc):
  *   - scores are softmax_scale * <q, k>; the workloads pre-scale q, scale = 1;
@@ -692,5 +695,101 @@ int64_t oracle_verify_tokens(const float *p, const float *q, const int32_t *x,
         n_acc[b] = j;
         n_bad += bad;
     }
+    return n_bad;
+}
+
+/* ======================================================================== */
+/* MagicDec draft attention: StreamingLLM over the target's own paged cache  */
+/* ======================================================================== */
+/*
+ * MagicDec drafts with the target model itself, attending to a sink +
+ * sliding-window subset of the target's KV cache, and (as in StreamingLLM)
+ * gives tokens their positions inside that reduced cache, not in the text
+ * (Section 3.1 footnote; Section 4: sink 1, window 64).
+ *
+ * Readings: the target cache holds keys already turned by their original
+ * position p (rotary, half-split pairs (d, d + D/2), angle p * theta^(-2d/D));
+ * t = ctx_lens[b] entries are visible to the current token, its own included;
+ * the visible positions are [0, s) and [w0, t) with s = min(n_sink, t) and
+ * w0 = max(s, t - window); their cache indices are c = p for p < s and
+ * c = s + (p - w0) otherwise, and the query's index is c_q = (number of
+ * visible entries) - 1.  Each key is turned by (c - p) to sit at its cache
+ * index and the (unrotated) query by c_q; both are rounded to bf16, as the
+ * model's operands are; values are not rotated.  theta = 0: no rotation.
+ * A length t < 1 or beyond the block table, or a page id outside the cache
+ * among the visible entries, gives NaN rows and is counted.
+ */
+static void rotate_pairs(const uint16_t *src, double delta, int32_t D,
+                         double theta, uint16_t *dst)
+{
+    for (int32_t d = 0; d < D / 2; ++d) {
+        double a0 = bf16_to_double(src[d]), a1 = bf16_to_double(src[d + D / 2]);
+        double r0 = a0, r1 = a1;
+        if (theta > 0.0 && delta != 0.0) {
+            double ang = delta * pow(theta, -2.0 * d / D);
+            double cs = cos(ang), sn = sin(ang);
+            r0 = a0 * cs - a1 * sn;
+            r1 = a1 * cs + a0 * sn;
+        }
+        dst[d] = double_to_bf16_bits(r0);
+        dst[d + D / 2] = double_to_bf16_bits(r1);
+    }
+}
+
+int64_t oracle_magicdec(const uint16_t *q, const uint16_t *k_cache,
+                        const uint16_t *v_cache, const int32_t *block_table,
+                        const int32_t *ctx_lens, int32_t B, int32_t Hq,
+                        int32_t Hkv, int32_t D, int32_t page_size,
+                        int32_t max_pages, int32_t num_pages, int32_t n_sink,
+                        int32_t window, double theta, double scale, double *out)
+{
+    if (B < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || D < 2 || D % 2 != 0 ||
+        page_size < 1 || n_sink < 0 || window < 1 || theta < 0.0)
+        return -1;
+    int64_t S = (int64_t)n_sink + window;
+    uint16_t *kc = (uint16_t *)malloc(sizeof(uint16_t) * (size_t)(S * D));
+    uint16_t *qe = (uint16_t *)malloc(sizeof(uint16_t) * (size_t)D);
+    const uint16_t **keys = (const uint16_t **)malloc(sizeof(*keys) * (size_t)S);
+    const uint16_t **vals = (const uint16_t **)malloc(sizeof(*vals) * (size_t)S);
+    double *scores = (double *)malloc(sizeof(double) * (size_t)S);
+    if (!kc || !qe || !keys || !vals || !scores) {
+        free(kc); free(qe); free(keys); free(vals); free(scores);
+        return -1;
+    }
+    int64_t n_bad = 0;
+    for (int32_t b = 0; b < B; ++b) {
+        int64_t t = ctx_lens[b];
+        int ok = t >= 1 && t <= (int64_t)max_pages * page_size;
+        int64_t s = ok ? (t < n_sink ? t : n_sink) : 0;
+        int64_t w0 = ok ? (t - window > s ? t - window : s) : 0;
+        int64_t n = s + (ok ? t - w0 : 0);
+        for (int64_t c = 0; ok && c < n; ++c) {
+            int64_t p = c < s ? c : w0 + (c - s);
+            int64_t page = block_table[(int64_t)b * max_pages + p / page_size];
+            if (page < 0 || page >= num_pages)
+                ok = 0;
+        }
+        for (int32_t h = 0; h < Hq; ++h) {
+            int32_t g = h / (Hq / Hkv);
+            double *o = out + ((int64_t)b * Hq + h) * D;
+            if (!ok) {
+                for (int32_t d = 0; d < D; ++d)
+                    o[d] = NAN;
+                continue;
+            }
+            for (int64_t c = 0; c < n; ++c) {
+                int64_t p = c < s ? c : w0 + (c - s);
+                int64_t page = block_table[(int64_t)b * max_pages + p / page_size];
+                int64_t row = ((page * Hkv + g) * page_size + p % page_size) * D;
+                rotate_pairs(k_cache + row, (double)(c - p), D, theta, kc + c * D);
+                keys[c] = kc + c * D;
+                vals[c] = v_cache + row;
+            }
+            rotate_pairs(q + ((int64_t)b * Hq + h) * D, (double)(n - 1), D, theta, qe);
+            attend(qe, keys, vals, n, D, scale, scores, o);
+        }
+        n_bad += !ok;
+    }
+    free(kc); free(qe); free(keys); free(vals); free(scores);
     return n_bad;
 }

@@ -653,4 +653,127 @@ def pin_tokens_invalid_inputs(lib):
     assert out[1].tolist() == [1, 2]
 
 
+# --------------------------------------------------------------------------
+# MagicDec draft attention pins
+# --------------------------------------------------------------------------
+def _rope_f64(x, pos, theta):
+    """Half-split rotary turn of x [..., D] (float64) by position pos, with
+    math.cos / math.sin / math.pow, the C library the oracle calls."""
+    D = x.shape[-1]
+    out = x.copy()
+    for d in range(D // 2):
+        a = pos * math.pow(theta, -2.0 * d / D)
+        c, s_ = math.cos(a), math.sin(a)
+        out[..., d] = x[..., d] * c - x[..., d + D // 2] * s_
+        out[..., d + D // 2] = x[..., d + D // 2] * c + x[..., d] * s_
+    return out
+
+
+def _md_case(rng, L, Hq, Hkv, D, shuffle=True):
+    B, T = len(L), int(max(L))
+    Kl = _f32_to_bf16_bits(rng.integers(-3, 4, size=(B, Hkv, T, D)).astype(np.float32))
+    Vl = _rand_bf16_bits(rng, (B, Hkv, T, D))
+    kc, vc, bt = _paged_from_logical(Kl, Vl, L, rng)
+    q = _rand_bf16_bits(rng, (B, Hq, D), scale=0.2)
+    return q, Kl, Vl, kc, vc, bt
+
+
+def pin_magicdec_without_rotation_is_sink_window(lib):
+    """theta = 0: exactly the sink + window attention of the draft definition
+    (the same visible set, read through the block table)."""
+    rng = np.random.default_rng(51)
+    L = np.array([1, 3, 66, 130, 200], dtype=np.int32)
+    q, Kl, Vl, kc, vc, bt = _md_case(rng, L, 4, 2, 16)
+    got, nb = oracle.magicdec(q, kc, vc, bt, L, 2, 64, 0.0, lib=lib)
+    want, nb2 = oracle.draft_logical(q, Kl, Vl, L, 2, 64, lib=lib)
+    assert nb == 0 and nb2 == 0
+    np.testing.assert_allclose(got, want, rtol=1e-14, atol=1e-14)
+
+
+def pin_magicdec_uniform_query_closed_form(lib):
+    """q = 0 (any rotation leaves it 0): the mean of the visible values; value
+    j carries its own position, so the mean is the closed form of the sink +
+    window positions."""
+    rng = np.random.default_rng(52)
+    L = np.array([1, 5, 70, 129, 250], dtype=np.int32)   # positions exact in bf16
+    n_sink, window, D = 3, 20, 8
+    q, Kl, _, _, _, _ = _md_case(rng, L, 2, 1, D)
+    q[:] = 0
+    T = int(L.max())
+    vals = np.zeros((len(L), 1, T, D), dtype=np.float32)
+    vals[..., 0] = np.arange(T)[None, None, :]
+    vals[..., 1] = 1.0
+    Vl = _f32_to_bf16_bits(vals)
+    kc, vc, bt = _paged_from_logical(Kl, Vl, L, rng)
+    got, nb = oracle.magicdec(q, kc, vc, bt, L, n_sink, window, 10000.0, lib=lib)
+    assert nb == 0
+    for b, t in enumerate(L):
+        np.testing.assert_allclose(got[b, :, 0], _draft_positions_closed_form(int(t), n_sink, window),
+                                   rtol=1e-12)
+        np.testing.assert_allclose(got[b, :, 1], 1.0, rtol=1e-14)
+
+
+def pin_magicdec_full_window_is_rotary_decoding(lib):
+    """window >= t: cache indices equal text positions, so keys keep their
+    stored rotation and the query turns by t - 1: plain rotary decoding
+    (the verify definition at k = 0 with that query)."""
+    rng = np.random.default_rng(53)
+    L = np.array([1, 7, 64, 100], dtype=np.int32)
+    theta, D = 10000.0, 16
+    q, _, _, kc, vc, bt = _md_case(rng, L, 4, 2, D)
+    got, nb = oracle.magicdec(q, kc, vc, bt, L, 1, 128, theta, lib=lib)
+    assert nb == 0
+    qf = _bits_to_f64(q)
+    qe = np.zeros_like(q)
+    for b, t in enumerate(L):
+        r = _rope_f64(qf[b], float(t - 1), theta)
+        qe[b] = np.array([[oracle.round_bf16(v, lib=lib) for v in row] for row in r],
+                         dtype=np.uint16)
+    want, nb2 = oracle.verify(qe[:, None], kc, vc, bt, L, 0, lib=lib)
+    assert nb2 == 0
+    np.testing.assert_allclose(got, want[:, 0], rtol=1e-13, atol=1e-13)
+
+
+def pin_magicdec_positions_are_cache_indices(lib):
+    """The same visible tokens (keys stored turned by their own text
+    positions) at two different context lengths give the same attention: only
+    positions inside the reduced cache matter.  Equal up to the bf16 rounding
+    of the stored and re-turned keys."""
+    rng = np.random.default_rng(54)
+    n_sink, window, D, Hkv, Hq, theta = 2, 12, 32, 1, 2, 10000.0
+    n = n_sink + window
+    kraw = rng.standard_normal((Hkv, n, D))
+    vraw = _rand_bf16_bits(rng, (Hkv, n, D))
+    q = _rand_bf16_bits(rng, (1, Hq, D), scale=0.7)
+    outs = []
+    for t in (40, 300):
+        Kl = np.zeros((1, Hkv, t, D), dtype=np.uint16)
+        Vl = np.zeros((1, Hkv, t, D), dtype=np.uint16)
+        pos = list(range(n_sink)) + list(range(t - window, t))
+        for c, p_ in enumerate(pos):
+            r = _rope_f64(kraw[:, c], float(p_), theta)
+            Kl[0, :, p_] = torch.from_numpy(r.astype(np.float32)).to(torch.bfloat16) \
+                .view(torch.int16).numpy().view(np.uint16)
+            Vl[0, :, p_] = vraw[:, c]
+        L = np.array([t], dtype=np.int32)
+        kc, vc, bt = _paged_from_logical(Kl, Vl, L, rng)
+        o, nb = oracle.magicdec(q, kc, vc, bt, L, n_sink, window, theta, lib=lib)
+        assert nb == 0
+        outs.append(o)
+    rel = np.linalg.norm(outs[0] - outs[1]) / np.linalg.norm(outs[1])
+    assert rel < 2e-2, rel
+
+
+def pin_magicdec_invalid(lib):
+    """t = 0, t beyond the table, or a visible page outside the cache: NaN."""
+    rng = np.random.default_rng(55)
+    L = np.array([0, 40, 40, 500], dtype=np.int32)
+    q, _, _, kc, vc, bt = _md_case(rng, np.array([1, 40, 40, 64]), 2, 1, 8)
+    bt = bt.copy()
+    bt[2, 0] = 99999
+    got, nb = oracle.magicdec(q, kc, vc, bt, L, 1, 8, 10000.0, lib=lib)
+    assert nb == 3
+    assert np.all(np.isnan(got[[0, 2, 3]])) and np.all(np.isfinite(got[1]))
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -69,6 +69,17 @@ MUTATIONS = [
     ("race_argmin", "if (key > best) {", "if (best == 0 || key < best) {"),
     ("accepted_tokens_reversed", "o[i] = x[(int64_t)b * k + i];",
      "o[i] = x[(int64_t)b * k + (j - 1 - i)];"),
+    ("magicdec_delta_sign", "rotate_pairs(k_cache + row, (double)(c - p), D, theta, kc + c * D);",
+     "rotate_pairs(k_cache + row, (double)(p - c), D, theta, kc + c * D);"),
+    ("magicdec_query_text_position",
+     "rotate_pairs(q + ((int64_t)b * Hq + h) * D, (double)(n - 1), D, theta, qe);",
+     "rotate_pairs(q + ((int64_t)b * Hq + h) * D, (double)(t - 1), D, theta, qe);"),
+    ("magicdec_window_start", "int64_t w0 = ok ? (t - window > s ? t - window : s) : 0;",
+     "int64_t w0 = ok ? (t - window + 1 > s ? t - window + 1 : s) : 0;"),
+    ("magicdec_no_sinks", "int64_t s = ok ? (t < n_sink ? t : n_sink) : 0;", "int64_t s = 0;"),
+    ("magicdec_pair_partner",
+     "double a0 = bf16_to_double(src[d]), a1 = bf16_to_double(src[d + D / 2]);",
+     "double a0 = bf16_to_double(src[d]), a1 = bf16_to_double(src[d ^ 1]);"),
 ]
 
 
