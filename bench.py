@@ -577,6 +577,37 @@ def spire_arm(args, cfg):
     tb = tokens_bytes(n_acc_h, k, V_tok)
     del ti
 
+    # ---- the MagicDec baseline's draft step: sink 1 + window 64 over the target's
+    # own paged cache (Section 4), positions inside the reduced cache
+    md_sink, md_win = 1, 64
+    md_ws = torch.empty(spire.spire_magicdec_workspace_bytes(vdesc, md_sink, md_win),
+                        dtype=torch.uint8, device=dev)
+    md_out = torch.empty(drafts[0].q.shape, dtype=torch.float32, device=dev)
+
+    def call_magicdec(j):
+        st = spire.spire_magicdec_attention(drafts[j].q, vi.k_cache, vi.v_cache, vi.block_table,
+                                            drafts[j].ctx_lens, md_sink, md_win, 10000.0, vdesc,
+                                            md_out, md_ws, md_ws.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_magicdec_attention")
+
+    for _ in range(max(3, args.warmup)):
+        call_magicdec(0)
+    torch.cuda.synchronize(dev)
+    md_ev = []
+    for s in range(a_steps):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call_magicdec(s % k)
+        b.record(stream)
+        md_ev.append((a, b))
+    torch.cuda.synchronize(dev)
+    md_ms = reduce_max([statistics.mean(a.elapsed_time(b) for a, b in md_ev)], dist, dev)[0]
+    md_bytes = statistics.mean(draft_bytes(wl.draft_ctx_for_step(L, k, j), md_sink + md_win, Hq,
+                                           Hkv, D) for j in range(k))
+    del md_ws
+
     if rank != 0:
         if dist is not None:
             dist.barrier()
@@ -629,6 +660,13 @@ def spire_arm(args, cfg):
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "launches": 3},
                    "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
+                   "magicdec_draft_step": {
+                       "what": "spire_magicdec_attention: sink %d + window %d over the target's "
+                               "paged cache, keys and query re-turned to cache positions "
+                               "(gather + draft attention launches)" % (md_sink, md_win),
+                       "us": md_ms * 1e3, "algorithmic_bytes": md_bytes,
+                       "gbs": md_bytes / (md_ms * 1e-3) / 1e9,
+                       "spire_draft_step_us": d_ms / k * 1e3},
                    "verify_tokens": {
                        "shape": "B=%d, k=%d, vocabulary %d (fp32 distributions)" % (B, k, V_tok),
                        "us": tok_ms * 1e3, "algorithmic_bytes": tb,

@@ -21,6 +21,9 @@
  *                                 token's activations into each layer's memory
  *                                 vector, project it to K/V and store it in
  *                                 the bounded cache (Section 3.3).
+ *   spire_magicdec_attention      the MagicDec baseline's draft attention:
+ *                                 sink + window over the target's own paged
+ *                                 cache, positions inside that reduced cache.
  *   spire_verify_tokens           the round's token verification: modified
  *                                 rejection sampling of the draft tokens
  *                                 (Section 1).
@@ -264,6 +267,48 @@ SPIRE_API spire_status spire_feedback_append(const void *x, const float *mix_w,
                                              const spire_append_desc *desc, void *kv,
                                              void *workspace, size_t ws_bytes,
                                              void *stream);
+
+/*
+ * MagicDec draft attention -- the paper's main baseline (Section 4): the
+ * target model drafts for itself, attending with a StreamingLLM mask (sink
+ * entries plus a sliding window; sink 1, window 64 in the paper) to its own
+ * paged KV cache, and, like StreamingLLM, gives entries their positions inside
+ * that reduced cache rather than in the text (Section 3.1, footnote).
+ *
+ * For sequence b with t = ctx_lens[b] visible cache entries (the current
+ * token's own included), the visible positions are [0, s) and [w0, t) with
+ * s = min(n_sink, t), w0 = max(s, t - window); entry p gets cache index c = p
+ * (sinks) or s + (p - w0) (window), and the query the last index, n - 1, with
+ * n the number of visible entries.  The target cache holds keys turned by
+ * their text position (rotary, half-split pairs (d, d + D/2), angle
+ * p * rope_theta^(-2d/D)); each visible key is turned by (c - p) and the
+ * query (given unrotated) by n - 1, both rounded to bf16, values unchanged;
+ * then softmax attention as spire_draft_sparse_attention.  rope_theta = 0
+ * skips every rotation.
+ *
+ *   q          bf16 [B, Hq, D], not rotated.
+ *   k_cache, v_cache, block_table: the target's paged cache as for
+ *              spire_verify_attention.
+ *   ctx_lens   int32 [B] on the device: 1 <= t <= max_pages_per_seq * 64.
+ *   n_sink >= 0, window >= 1, n_sink + window <= 65536.
+ *   out        fp32 [B, Hq, D].
+ *   workspace  >= spire_magicdec_workspace_bytes(desc, n_sink, window) bytes:
+ *              the reduced cache, the turned queries and the attention's own
+ *              workspace.
+ * A length out of range, or a block-table entry outside the cache among the
+ * visible entries, gives NaN rows and sets SPIRE_DEVERR_CTX_LEN.
+ */
+SPIRE_API size_t spire_magicdec_workspace_bytes(const spire_attn_desc *desc, int32_t n_sink,
+                                                int32_t window);
+
+SPIRE_API spire_status spire_magicdec_attention(const void *q, const void *k_cache,
+                                                const void *v_cache,
+                                                const int32_t *block_table,
+                                                const int32_t *ctx_lens, int32_t n_sink,
+                                                int32_t window, float rope_theta,
+                                                const spire_attn_desc *desc, float *out,
+                                                void *workspace, size_t ws_bytes,
+                                                void *stream);
 
 /*
  * Token verification of a speculation round (modified rejection sampling).

@@ -13,6 +13,8 @@ libspire (include/spire.h):
   spire_feedback_append          the draft step's cache update: per-layer
                                  memory vector, K/V projection, bounded-cache
                                  slot (Section 3.3)
+  spire_magicdec_attention       the MagicDec baseline's draft attention over
+                                 the target's own cache (Section 3.1 footnote)
   spire_verify_tokens            token verification: modified rejection
                                  sampling of the round's drafts (Section 1)
 
@@ -27,7 +29,8 @@ from . import _lib
 from ._lib import (SpireError, make_append_desc, make_desc, spire_draft_slot,
                    spire_draft_sparse_attention, spire_draft_workspace_bytes,
                    spire_feedback_append, spire_feedback_append_workspace_bytes,
-                   spire_get_device_error, spire_status_string, spire_verify_attention,
+                   spire_get_device_error, spire_magicdec_attention,
+                   spire_magicdec_workspace_bytes, spire_status_string, spire_verify_attention,
                    spire_verify_attention_noalloc, spire_verify_tokens,
                    spire_verify_tokens_workspace_bytes, spire_verify_workspace_bytes)
 
@@ -35,7 +38,8 @@ __all__ = [
     "SpireError", "make_desc", "make_append_desc", "spire_verify_attention",
     "spire_verify_attention_noalloc", "spire_draft_sparse_attention", "spire_feedback_append",
     "spire_feedback_append_workspace_bytes", "feedback_append", "spire_verify_tokens",
-    "spire_verify_tokens_workspace_bytes", "verify_tokens",
+    "spire_verify_tokens_workspace_bytes", "verify_tokens", "spire_magicdec_attention",
+    "spire_magicdec_workspace_bytes", "magicdec_attention",
     "spire_verify_workspace_bytes", "spire_draft_workspace_bytes", "spire_draft_slot",
     "spire_get_device_error", "spire_status_string", "verify_attention", "draft_attention",
     "verify_desc", "draft_desc",
@@ -127,3 +131,22 @@ def verify_tokens(p, q, draft_tokens, u, e, workspace=None, stream=None):
     if st != 0:
         raise SpireError(st, "spire_verify_tokens")
     return out, n_acc
+
+
+def magicdec_attention(q, k_cache, v_cache, block_table, ctx_lens, n_sink, window, rope_theta,
+                       softmax_scale=1.0, out=None, workspace=None, stream=None):
+    """MagicDec draft attention over the target's paged cache; q bf16
+    [B, Hq, D] (not rotated).  Returns out fp32 [B, Hq, D]."""
+    B, Hq, D = q.shape
+    desc = make_desc(B, Hq, k_cache.shape[1], D, k_cache.shape[2], block_table.shape[1],
+                     k_cache.shape[0], softmax_scale)
+    ws_bytes = spire_magicdec_workspace_bytes(desc, n_sink, window)
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=q.device)
+    st = spire_magicdec_attention(q, k_cache, v_cache, block_table, ctx_lens, n_sink, window,
+                                  rope_theta, desc, out, workspace, workspace.numel(), stream)
+    if st != 0:
+        raise SpireError(st, "spire_magicdec_attention")
+    return out

@@ -37,6 +37,8 @@ EXPORTED = (
     "spire_draft_sparse_attention",
     "spire_feedback_append_workspace_bytes",
     "spire_feedback_append",
+    "spire_magicdec_workspace_bytes",
+    "spire_magicdec_attention",
     "spire_verify_tokens_workspace_bytes",
     "spire_verify_tokens",
     "spire_draft_slot",
@@ -100,6 +102,11 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_feedback_append_workspace_bytes.argtypes = [A]
     lib.spire_feedback_append.restype = ctypes.c_int
     lib.spire_feedback_append.argtypes = [P, P, P, P, A, P, P, SZ, P]
+    lib.spire_magicdec_workspace_bytes.restype = SZ
+    lib.spire_magicdec_workspace_bytes.argtypes = [D, I32, I32]
+    lib.spire_magicdec_attention.restype = ctypes.c_int
+    lib.spire_magicdec_attention.argtypes = [P, P, P, P, P, I32, I32, ctypes.c_float, D, P, P, SZ,
+                                             P]
     lib.spire_verify_tokens_workspace_bytes.restype = SZ
     lib.spire_verify_tokens_workspace_bytes.argtypes = [I32, I32, I32]
     lib.spire_verify_tokens.restype = ctypes.c_int
@@ -193,6 +200,18 @@ def spire_feedback_append(x, mix_w, w_kv, pos, desc, kv, workspace, ws_bytes, st
     return int(LIB.spire_feedback_append(
         _ptr(x), _ptr(mix_w), _ptr(w_kv), _ptr(pos), _desc_ref(desc), _ptr(kv), _ptr(workspace),
         int(ws_bytes), _stream(stream, x)))
+
+
+def spire_magicdec_workspace_bytes(desc: spire_attn_desc, n_sink: int, window: int) -> int:
+    return int(LIB.spire_magicdec_workspace_bytes(_desc_ref(desc), int(n_sink), int(window)))
+
+
+def spire_magicdec_attention(q, k_cache, v_cache, block_table, ctx_lens, n_sink, window,
+                             rope_theta, desc, out, workspace, ws_bytes, stream=None) -> int:
+    return int(LIB.spire_magicdec_attention(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(ctx_lens), int(n_sink),
+        int(window), float(rope_theta), _desc_ref(desc), _ptr(out), _ptr(workspace),
+        int(ws_bytes), _stream(stream, q)))
 
 
 def spire_verify_tokens_workspace_bytes(batch: int, k: int, vocab: int) -> int:

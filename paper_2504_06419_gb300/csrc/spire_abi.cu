@@ -169,6 +169,133 @@ __global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n)
     for (int i = threadIdx.x; i < n; i += blockDim.x) cnt[i] = 0;
 }
 
+// ------------------------------------------------------------- MagicDec gather
+// MagicDec's draft attends, with positions inside the reduced cache, to the
+// sink + window entries of the target's own paged cache (Section 3.1
+// footnote).  This kernel builds that reduced cache: one warp per row.
+//   sequence rows  n_vis[b] = number of visible entries (0 if t is out of
+//                  range or a visible page id is outside the cache)
+//   K / V rows     entry c of (b, g): the text position p, K turned by
+//                  (c - p) (rotary pairs (d, d + D/2)) and rounded to bf16,
+//                  V copied
+//   query rows     q turned by the query's cache index n_vis - 1
+// Angles: (c - p) * freq[d] and its reduction modulo 2 pi in double, sine and
+// cosine of the reduced angle in fp32 (positions up to 2^31 keep their
+// accuracy).
+struct MdParams {
+    const __nv_bfloat16* q;        // [B, Hq, D], not rotated
+    const __nv_bfloat16* k_cache;  // [num_pages, Hkv, 64, D], keys turned by text position
+    const __nv_bfloat16* v_cache;
+    const int32_t* block_table;
+    const int32_t* ctx_lens;
+    __nv_bfloat16* kv;             // [B, 2, Hkv, S, D] reduced cache
+    __nv_bfloat16* q_eff;          // [B, Hq, D]
+    int32_t* n_vis;                // [B]
+    int B, Hq, Hkv, D, S, n_sink, window, max_pages, num_pages, rotate;
+    double freq[64];
+};
+
+struct MdVisible {
+    int s, w0, n;
+};
+
+__device__ __forceinline__ MdVisible md_visible(const MdParams& p, int t) {
+    MdVisible v{0, 0, 0};
+    if (t < 1 || (long long)t > (long long)p.max_pages * kPage) return v;
+    v.s = t < p.n_sink ? t : p.n_sink;
+    v.w0 = t - p.window > v.s ? t - p.window : v.s;
+    v.n = v.s + (t - v.w0);
+    return v;
+}
+
+// turn pairs (d, d + D/2) of a row by delta positions (lane handles d = lane + 32 i)
+__device__ __forceinline__ void md_rotate_row(const __nv_bfloat16* src, __nv_bfloat16* dst,
+                                              long long delta, const MdParams& p, int lane) {
+    const int half = p.D / 2;
+    const double kTwoPi = 6.283185307179586476925286766559;
+    const double kInvTwoPi = 0.15915494309189533576888376337251;
+    for (int d = lane; d < half; d += 32) {
+        const float a0 = __bfloat162float(src[d]), a1 = __bfloat162float(src[d + half]);
+        float r0 = a0, r1 = a1;
+        if (p.rotate && delta != 0) {
+            const double ang = (double)delta * p.freq[d];
+            const double red = fma(-kTwoPi, rint(ang * kInvTwoPi), ang);
+            float sn, cs;
+            sincosf((float)red, &sn, &cs);
+            r0 = a0 * cs - a1 * sn;
+            r1 = a1 * cs + a0 * sn;
+        }
+        dst[d] = __float2bfloat16_rn(r0);
+        dst[d + half] = __float2bfloat16_rn(r1);
+    }
+}
+
+__global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) {
+    const int lane = threadIdx.x & 31;
+    const long long n_kv = (long long)p.B * p.Hkv * p.S;
+    const long long total = p.B + n_kv + (long long)p.B * p.Hq;
+    for (long long item = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5; item < total;
+         item += ((long long)gridDim.x * blockDim.x) >> 5) {
+        if (item < p.B) {
+            // sequence row: the visible count, after checking every visible page
+            const int b = (int)item;
+            MdVisible v = md_visible(p, p.ctx_lens[b]);
+            bool ok = v.n > 0;
+            const int t = p.ctx_lens[b];
+            const int pg_s = v.s > 0 ? (v.s - 1) / kPage + 1 : 0;     // pages of the sinks
+            const int pg_w0 = v.w0 / kPage, pg_w1 = ok ? (t - 1) / kPage : -1;
+            for (int pg = lane; ok && pg < pg_s; pg += 32) {
+                const int id = p.block_table[(long long)b * p.max_pages + pg];
+                if (id < 0 || id >= p.num_pages) ok = false;
+            }
+            for (int pg = pg_w0 + lane; ok && pg <= pg_w1; pg += 32) {
+                const int id = p.block_table[(long long)b * p.max_pages + pg];
+                if (id < 0 || id >= p.num_pages) ok = false;
+            }
+            ok = __all_sync(0xffffffffu, ok);
+            if (lane == 0) p.n_vis[b] = ok ? v.n : 0;
+        } else if (item < p.B + n_kv) {
+            long long r = item - p.B;
+            const int c = (int)(r % p.S); r /= p.S;
+            const int g = (int)(r % p.Hkv);
+            const int b = (int)(r / p.Hkv);
+            const MdVisible v = md_visible(p, p.ctx_lens[b]);
+            if (c >= v.n) continue;
+            const int pos = c < v.s ? c : v.w0 + (c - v.s);
+            const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
+            if (id < 0 || id >= p.num_pages) continue;   // the sequence row reports it
+            const long long src = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * p.D;
+            const long long dk = ((((long long)b * 2 + 0) * p.Hkv + g) * p.S + c) * p.D;
+            const long long dv = ((((long long)b * 2 + 1) * p.Hkv + g) * p.S + c) * p.D;
+            md_rotate_row(p.k_cache + src, p.kv + dk, (long long)c - pos, p, lane);
+            for (int d = 2 * lane; d < p.D; d += 64)
+                *reinterpret_cast<__nv_bfloat162*>(p.kv + dv + d) =
+                    *reinterpret_cast<const __nv_bfloat162*>(p.v_cache + src + d);
+        } else {
+            const long long r = item - p.B - n_kv;
+            const int b = (int)(r / p.Hq);
+            const MdVisible v = md_visible(p, p.ctx_lens[b]);
+            if (v.n == 0) continue;
+            md_rotate_row(p.q + r * p.D, p.q_eff + r * p.D, v.n - 1, p, lane);
+        }
+    }
+}
+
+struct MdLayout {
+    size_t draft, kv, q, nvis, total;
+};
+
+MdLayout md_layout(const spire_attn_desc* d, int S) {
+    MdLayout l{};
+    l.draft = 0;
+    size_t off = ws_layout(d->batch, d->num_kv_heads, rows_per_kv_head(d, 1), d->head_dim).total;
+    l.kv = off;   off += align256((size_t)d->batch * 2 * d->num_kv_heads * S * d->head_dim * 2);
+    l.q = off;    off += align256((size_t)d->batch * d->num_q_heads * d->head_dim * 2);
+    l.nvis = off; off += align256((size_t)d->batch * 4);
+    l.total = off;
+    return l;
+}
+
 // Shared launch sequence for both calls.
 spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorMap& tv,
                  const int32_t* block_table, const int32_t* ctx_lens, int kp1,
@@ -305,6 +432,81 @@ spire_status spire_draft_sparse_attention(const void* q, const void* kv, const i
     if (!encode_kv_map(&tkv, kv, desc->head_dim, uint64_t(S), planes)) return SPIRE_ERR_CUDA;
     return run(kModeDraft, q, tkv, tkv, nullptr, ctx_lens, 1, desc, int(S), out, workspace,
                static_cast<cudaStream_t>(stream));
+}
+
+size_t spire_magicdec_workspace_bytes(const spire_attn_desc* desc, int32_t n_sink,
+                                      int32_t window) {
+    if (check_common(desc) != SPIRE_OK || n_sink < 0 || window < 1 ||
+        (long long)n_sink + window > 65536)
+        return 0;
+    return md_layout(desc, n_sink + window).total;
+}
+
+spire_status spire_magicdec_attention(const void* q, const void* k_cache, const void* v_cache,
+                                      const int32_t* block_table, const int32_t* ctx_lens,
+                                      int32_t n_sink, int32_t window, float rope_theta,
+                                      const spire_attn_desc* desc, float* out, void* workspace,
+                                      size_t ws_bytes, void* stream) {
+    spire_status st = check_common(desc);
+    if (st != SPIRE_OK) return st;
+    if (n_sink < 0 || window < 1 || !std::isfinite(rope_theta) || rope_theta < 0.f)
+        return SPIRE_ERR_INVALID_ARG;
+    if ((long long)n_sink + window > 65536) return SPIRE_ERR_UNSUPPORTED;
+    if (desc->page_size != kPage) return SPIRE_ERR_UNSUPPORTED;
+    if (desc->max_pages_per_seq < 1 || desc->num_pages < 1) return SPIRE_ERR_INVALID_ARG;
+    if (rows_per_kv_head(desc, 1) > SPIRE_MAX_ROWS_PER_KV_HEAD) return SPIRE_ERR_UNSUPPORTED;
+    if ((long long)desc->num_pages * desc->num_kv_heads >= (1LL << 31) ||
+        (long long)desc->batch * desc->max_pages_per_seq >= (1LL << 31) ||
+        (long long)desc->max_pages_per_seq * kPage >= (1LL << 31) ||
+        (long long)desc->batch * 2 * desc->num_kv_heads >= (1LL << 31))
+        return SPIRE_ERR_UNSUPPORTED;
+    if (desc->batch == 0) return SPIRE_OK;
+    if (!q || !k_cache || !v_cache || !block_table || !ctx_lens || !out)
+        return SPIRE_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+        !aligned(block_table, 4) || !aligned(ctx_lens, 4))
+        return SPIRE_ERR_INVALID_ARG;
+    const int S = n_sink + window;
+    const MdLayout l = md_layout(desc, S);
+    if (!workspace || !aligned(workspace, 256) || ws_bytes < l.total) return SPIRE_ERR_WORKSPACE;
+    DeviceInfo di;
+    st = device_info(&di);
+    if (st != SPIRE_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    char* ws = static_cast<char*>(workspace);
+
+    MdParams mp{};
+    mp.q = static_cast<const __nv_bfloat16*>(q);
+    mp.k_cache = static_cast<const __nv_bfloat16*>(k_cache);
+    mp.v_cache = static_cast<const __nv_bfloat16*>(v_cache);
+    mp.block_table = block_table;
+    mp.ctx_lens = ctx_lens;
+    mp.kv = reinterpret_cast<__nv_bfloat16*>(ws + l.kv);
+    mp.q_eff = reinterpret_cast<__nv_bfloat16*>(ws + l.q);
+    mp.n_vis = reinterpret_cast<int32_t*>(ws + l.nvis);
+    mp.B = desc->batch;
+    mp.Hq = desc->num_q_heads;
+    mp.Hkv = desc->num_kv_heads;
+    mp.D = desc->head_dim;
+    mp.S = S;
+    mp.n_sink = n_sink;
+    mp.window = window;
+    mp.max_pages = desc->max_pages_per_seq;
+    mp.num_pages = desc->num_pages;
+    mp.rotate = rope_theta > 0.f;
+    // the rotary frequencies theta^(-2d/D): per-call constants, in double
+    for (int d = 0; d < desc->head_dim / 2; ++d)
+        mp.freq[d] = mp.rotate ? std::pow((double)rope_theta, -2.0 * d / desc->head_dim) : 0.0;
+    const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * S + mp.Hq);
+    long long blocks = (items * 32 + 255) / 256;
+    if (blocks > 32LL * di.sms) blocks = 32LL * di.sms;
+    magicdec_gather_kernel<<<(unsigned)blocks, 256, 0, s>>>(mp);
+    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+
+    CUtensorMap tkv;
+    const uint64_t planes = uint64_t(desc->batch) * 2u * uint64_t(desc->num_kv_heads);
+    if (!encode_kv_map(&tkv, mp.kv, desc->head_dim, uint64_t(S), planes)) return SPIRE_ERR_CUDA;
+    return run(kModeDraft, mp.q_eff, tkv, tkv, nullptr, mp.n_vis, 1, desc, S, out, workspace, s);
 }
 
 int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {

@@ -30,6 +30,7 @@ def test_header_declares_the_boundary():
         "spire_verify_attention_noalloc", "spire_draft_workspace_bytes", "spire_draft_sparse_attention", "spire_draft_slot",
         "spire_feedback_append_workspace_bytes", "spire_feedback_append",
         "spire_verify_tokens_workspace_bytes", "spire_verify_tokens",
+        "spire_magicdec_workspace_bytes", "spire_magicdec_attention",
         "spire_get_device_error", "spire_status_string"]), names
 
 
@@ -200,3 +201,27 @@ def test_tokens_workspace_and_host_checks(spire):
     assert call(ws_bytes=ws - 1) == E.SPIRE_ERR_WORKSPACE
     assert call(k=40) == E.SPIRE_ERR_UNSUPPORTED
     assert call(batch=0) == E.SPIRE_ERR_INVALID_ARG
+
+
+def test_magicdec_host_checks(spire):
+    E = spire._lib
+    d = _desc(spire)
+    ws = spire.spire_magicdec_workspace_bytes(d, 1, 64)
+    assert ws > spire.spire_draft_workspace_bytes(d, 1, 64)
+    assert spire.spire_magicdec_workspace_bytes(d, -1, 64) == 0
+    assert spire.spire_magicdec_workspace_bytes(d, 1, 0) == 0
+    good = 1 << 20
+    call = lambda **kw: spire.spire_magicdec_attention(**{**dict(
+        q=good, k_cache=good, v_cache=good, block_table=good, ctx_lens=good, n_sink=1,
+        window=64, rope_theta=10000.0, desc=d, out=good, workspace=good, ws_bytes=ws,
+        stream=0), **kw})
+    for name in ("q", "k_cache", "v_cache", "block_table", "ctx_lens", "out"):
+        assert call(**{name: 0}) == E.SPIRE_ERR_INVALID_ARG, name
+    assert call(workspace=0) == E.SPIRE_ERR_WORKSPACE
+    assert call(ws_bytes=ws - 1) == E.SPIRE_ERR_WORKSPACE
+    assert call(rope_theta=-1.0) == E.SPIRE_ERR_INVALID_ARG
+    assert call(rope_theta=float("nan")) == E.SPIRE_ERR_INVALID_ARG
+    assert call(window=0) == E.SPIRE_ERR_INVALID_ARG
+    assert call(q=good + 8) == E.SPIRE_ERR_INVALID_ARG
+    assert call(desc=_desc(spire, page_size=32)) == E.SPIRE_ERR_UNSUPPORTED
+    assert call(window=70000) == E.SPIRE_ERR_UNSUPPORTED
