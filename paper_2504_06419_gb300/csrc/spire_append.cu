@@ -10,9 +10,7 @@
 //   append_mix_kernel       m[i, b, :] in fp32 from x and softmax(w_i), stored
 //                           as two bf16 arrays m_hi = bf16(m), m_lo =
 //                           bf16(m - m_hi) in the workspace (~16 significant
-//                           bits together); block 0 instead writes the rotary
-//                           frequencies theta^(-2d/D) (double) and clears the
-//                           device error word.
+//                           bits together); clears the device error word.
 //   append_gemm_kernel      tcgen05 GEMM, split over K.  CTA (i, 128-row block
 //                           of W_i, token block of N, K range) accumulates
 //                           W_i[rows, K range] . m[tokens, K range]^T in tensor
@@ -33,6 +31,12 @@
 //                           reduced angle in fp32), rounds to bf16 and writes
 //                           the slot.  A negative position writes nothing and
 //                           sets the device error word.
+//
+// The GEMM and the finalize are launched with programmatic dependent launch:
+// their prologues overlap the kernel before them, and they wait
+// (griddepcontrol.wait) only before reading what it wrote.  The rotary
+// frequencies theta^(-2d/D) are per-call constants computed on the host in
+// double and passed to the finalize.
 //
 // The weights are read once (the only large operand: n_dl * F * d_model * 2
 // bytes); m (2 * n_dl * B * d_model * 2 bytes) is re-read from L2 by every row
@@ -63,11 +67,9 @@ struct AppendMixParams {
     const __nv_bfloat16* x;   // [n_act, B, d_model]
     const float* mix_w;       // [n_dl, n_act]
     __nv_bfloat16* m;         // [2 (hi, lo), n_dl, B, d_model]
-    double* freq;             // [D/2]
     int32_t* header;          // header[0] = number of error words
     int32_t* err;
-    int B, n_act, n_dl, d_model, half;
-    double theta;
+    int B, n_act, n_dl, d_model;
 };
 
 struct AppendGemmParams {
@@ -79,10 +81,10 @@ struct AppendGemmParams {
 struct AppendFinalParams {
     const float* part;
     const int32_t* pos;
-    const double* freq;
     __nv_bfloat16* kv;        // [n_dl, B, 2, Hkv, S, D]
     int32_t* err;
     int B, n_dl, F, Hkv, D, S, n_sink, window, ksplit, rotate;
+    double freq[64];          // theta^(-2d/D), d < D/2
 };
 
 // Shared-memory layout of one stage: the W tile, then the m_hi and m_lo tiles
@@ -92,16 +94,10 @@ __host__ __device__ constexpr int stage_bytes(int N) { return kATile + 2 * N * 1
 
 __global__ void __launch_bounds__(256) append_mix_kernel(const AppendMixParams p) {
     __shared__ float a[16 * 16];                 // softmax(w_i), [n_dl][n_act]
-    if (blockIdx.x == 0) {
-        // block 0: the rotary frequencies (double pow is slow here, so no other work
-        // waits for it) and the device error word
-        for (int d = threadIdx.x; d < p.half; d += blockDim.x)
-            p.freq[d] = pow(p.theta, -2.0 * d / (2 * p.half));
-        if (threadIdx.x == 0) {
-            p.header[0] = 1;
-            p.err[0] = 0;
-        }
-        return;
+    grid_dep_launch_dependents();                // the GEMM may start its prologue
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        p.header[0] = 1;
+        p.err[0] = 0;
     }
     if (threadIdx.x < p.n_dl) {
         const int i = threadIdx.x;
@@ -119,8 +115,8 @@ __global__ void __launch_bounds__(256) append_mix_kernel(const AppendMixParams p
     const int c8 = p.d_model / 8;                // 8-column groups per row
     const long long total = (long long)p.n_dl * p.B * c8;
     const long long plane = (long long)p.n_dl * p.B * p.d_model;
-    for (long long idx = (blockIdx.x - 1) * (long long)blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)(gridDim.x - 1) * blockDim.x) {
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
         const int c = (int)(idx % c8);
         const long long ib = idx / c8;           // i * B + b
         const int b = (int)(ib % p.B), i = (int)(ib / p.B);
@@ -196,6 +192,9 @@ __global__ void __launch_bounds__(kAppendThreads, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
     uint32_t err = 0;
+    grid_dep_launch_dependents();                // the finalize may start its prologue
+    // m and the cleared error word come from the mix kernel
+    grid_dep_wait();
 
     if (warp == 0) {
         // ------------------------------------------------ W, m_hi, m_lo tiles by TMA
@@ -284,6 +283,7 @@ __global__ void __launch_bounds__(kAppendThreads, 1)
 }
 
 __global__ void __launch_bounds__(64) append_finalize_kernel(const AppendFinalParams p) {
+    grid_dep_wait();                             // the GEMM's partials
     const int half = p.D / 2, q4 = half / 4;     // four pairs (d .. d + 3, + D/2) per thread
     const double kTwoPi = 6.283185307179586476925286766559;
     const double kInvTwoPi = 0.15915494309189533576888376337251;
@@ -381,9 +381,9 @@ bool plan_append(const spire_append_desc* d, AppendPlan* pl) {
     return true;
 }
 
-// workspace: header word | error word | rotary frequencies | m_hi, m_lo | partials
+// workspace: header word | error word | (reserved) | m_hi, m_lo | partials
 constexpr size_t kAppendHeader = 512;
-constexpr size_t kAppendFreq = 512;              // D/2 <= 64 doubles
+constexpr size_t kAppendFreq = 512;
 
 size_t append_m_bytes(const spire_append_desc* d) {
     return (((size_t)2 * d->num_draft_layers * d->batch * d->d_model * 2) + 255) & ~size_t(255);
@@ -447,19 +447,16 @@ spire_status spire_feedback_append(const void* x, const float* mix_w, const void
     mp.x = static_cast<const __nv_bfloat16*>(x);
     mp.mix_w = mix_w;
     mp.m = mbuf;
-    mp.freq = reinterpret_cast<double*>(ws + kAppendHeader);
     mp.header = reinterpret_cast<int32_t*>(ws);
     mp.err = reinterpret_cast<int32_t*>(ws + 256);
     mp.B = B;
     mp.n_act = desc->num_act;
     mp.n_dl = n_dl;
     mp.d_model = desc->d_model;
-    mp.half = desc->head_dim / 2;
-    mp.theta = (double)desc->rope_theta;
     const long long mix_items = (long long)n_dl * B * (desc->d_model / 8);
     long long mblocks = (mix_items + 255) / 256;
     if (mblocks > 8LL * sms) mblocks = 8LL * sms;
-    append_mix_kernel<<<(unsigned)(mblocks + 1), 256, 0, st>>>(mp);   // + block 0
+    append_mix_kernel<<<(unsigned)mblocks, 256, 0, st>>>(mp);
     if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
 
     AppendGemmParams gp{};
@@ -490,13 +487,17 @@ spire_status spire_feedback_append(const void* x, const float* mix_w, const void
             }
         }
     }
-    append_gemm_kernel<<<(unsigned)(tiles * ks), kAppendThreads, smem, st>>>(tw, tm, gp);
-    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+    if (launch_dependent(append_gemm_kernel, dim3((unsigned)(tiles * ks)), dim3(kAppendThreads),
+                         smem, st, tw, tm, gp) != cudaSuccess)
+        return SPIRE_ERR_CUDA;
 
     AppendFinalParams fp{};
     fp.part = gp.part;
     fp.pos = pos;
-    fp.freq = mp.freq;
+    for (int d = 0; d < desc->head_dim / 2; ++d)     // the same libm pow as the definition
+        fp.freq[d] = desc->rope_theta > 0.f
+                         ? std::pow((double)desc->rope_theta, -2.0 * d / desc->head_dim)
+                         : 0.0;
     fp.kv = static_cast<__nv_bfloat16*>(kv);
     fp.err = mp.err;
     fp.B = B;
@@ -513,8 +514,10 @@ spire_status spire_feedback_append(const void* x, const float* mix_w, const void
     // small blocks so that the few threads reach every SM
     long long blocks = (total + 63) / 64;
     if (blocks > 16LL * sms) blocks = 16LL * sms;
-    append_finalize_kernel<<<(unsigned)blocks, 64, 0, st>>>(fp);
-    return cudaGetLastError() == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
+    return launch_dependent(append_finalize_kernel, dim3((unsigned)blocks), dim3(64), 0, st, fp) ==
+                   cudaSuccess
+               ? SPIRE_OK
+               : SPIRE_ERR_CUDA;
 }
 
 }  // extern "C"

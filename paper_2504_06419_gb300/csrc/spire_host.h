@@ -5,6 +5,7 @@
 #include <cstdint>
 
 #include <cuda.h>
+#include <cuda_runtime.h>
 
 #include "spire.h"
 
@@ -20,5 +21,25 @@ spire_status host_device_info(int* sms, int* smem_optin);
 // box_inner x box_outer boxes with 128-byte swizzle.
 bool encode_2d_bf16_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                         uint32_t box_inner, uint32_t box_outer);
+
+// Launch a kernel with programmatic dependent launch: it may start while the
+// kernel before it in the stream runs (after that kernel's blocks have all
+// called griddepcontrol.launch_dependents or exited); the launched kernel
+// must execute griddepcontrol.wait before it reads anything that kernel wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t stream, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
 
 }  // namespace spire
