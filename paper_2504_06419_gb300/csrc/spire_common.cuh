@@ -91,7 +91,8 @@ __device__ __forceinline__ long long range_lo(int c, long long W, int N) {
 
 struct SchedShared {
     long long W, lo, hi, p0;   // total tiles, this CTA's range, first tile of sequence b0
-    int b0;
+    long long p1;              // first unit of sequence b1, which holds unit hi - 1
+    int b0, b1;
     int N;                     // CTAs with work: min(grid, W), so no range is empty
     int bad_len;               // some ctx_lens entry breaks the rules
     long long warp_sums[32];
@@ -149,6 +150,7 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
     const long long lo = c < N ? range_lo(c, W, N) : W, hi = c < N ? range_lo(c + 1, W, N) : W;
     if (threadIdx.x == 0) {
         sh->W = W; sh->lo = lo; sh->hi = hi; sh->b0 = 0; sh->p0 = 0; sh->N = N;
+        sh->b1 = 0; sh->p1 = 0;
         sh->bad_len = any_bad;
     }
     long long carry = 0;
@@ -163,6 +165,10 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
             sh->b0 = b;
             sh->p0 = P * p.Hkv;
         }
+        if (b < p.B && lo < hi && P * p.Hkv <= hi - 1 && hi - 1 < (P + U) * p.Hkv) {
+            sh->b1 = b;
+            sh->p1 = P * p.Hkv;
+        }
         carry += chunk;
     }
     __syncthreads();
@@ -174,31 +180,60 @@ struct TileMeta {
     int flags, slot, nseg, first_slot;
 };
 
-// Walks the tiles of this CTA's unit range in order, tracking (b, g, t)
-// incrementally and stepping over head units; the segment bookkeeping
-// (divisions) runs once per segment, not per tile.
+// Walks the tiles of this CTA's unit range, tracking (b, g, t) incrementally
+// and stepping over head units; the segment bookkeeping (slot, number of
+// segments, first slot) is computed once per segment.  With tail_first, when
+// the range ends inside a pair that continues in the next CTA, that pair's
+// segment is walked first and then the rest of the range from its start: the
+// pair's two halves are then done near the start of both CTAs, so its merge
+// overlaps the remaining work instead of trailing the kernel (used by the
+// warp-MMA kernel, whose short draft ranges end in such a merge; measured
+// slower for the tcgen05 kernel, whose softmax warps do the merge).  Segments,
+// slots and the tiles of each segment are the same in either order.
 struct TileWalker {
-    long long x, hi, lo, W;    // unit of the next tile, end / start of range, total units
+    long long x, end, lo, W;   // unit of the next tile, end of the current part, range start
+    long long rest_end;        // end of the second part (the tail pair's first unit), or -1
     int N;
     int b, g, t, T, leff;      // current sequence / KV head / tile-in-pair, tiles per pair
     bool valid, first;
     int slot, nseg, first_slot;
+    int b0;
+    long long p0;
 
-    __device__ void init(const AttnParams& p, const SchedShared& sh) {
-        x = sh.lo; hi = sh.hi; lo = sh.lo; W = sh.W; N = sh.N;
-        b = sh.b0; g = 0; t = 0; T = 1; leff = 0; valid = false; first = true;
+    // decode the pair and tile at unit x of sequence b (first unit pb)
+    __device__ void seek(const AttnParams& p, long long at, int sb, long long pb) {
+        x = at; b = sb; g = 0; t = 0; first = true;
+        T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
+        const long long off = x - pb;
+        const int U = T + kHead;
+        g = (int)(off / U);
+        const int u = (int)(off - (long long)g * U);
+        if (u < kHead) x += kHead - u;             // a part starting in a pair's head
+        else t = u - kHead;
+    }
+
+    __device__ void init(const AttnParams& p, const SchedShared& sh, bool tail_first) {
+        lo = sh.lo; W = sh.W; N = sh.N; b0 = sh.b0; p0 = sh.p0;
         slot = nseg = first_slot = 0;
-        if (x < hi) {
-            T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
-            const long long off = x - sh.p0;
-            const int U = T + kHead;
-            g = (int)(off / U);
-            const int u = (int)(off - (long long)g * U);
-            if (u < kHead) x += kHead - u;         // range starts in a pair's head
-            else t = u - kHead;
+        valid = false; T = 1; leff = 0; b = sh.b0; g = 0; t = 0; first = true;
+        rest_end = -1;
+        x = sh.lo; end = sh.hi;
+        if (sh.lo >= sh.hi) return;
+        // the pair holding the range's last unit
+        int le1;
+        bool ok1;
+        const int T1 = seq_tiles(p, p.ctx_lens[sh.b1], &le1, &ok1);
+        const int U1 = T1 + kHead;
+        const long long g1 = (sh.hi - 1 - sh.p1) / U1;
+        const long long pstart = sh.p1 + g1 * U1;
+        if (tail_first && pstart > sh.lo && sh.hi - 1 - pstart >= kHead && pstart + U1 > sh.hi) {
+            seek(p, pstart + kHead, sh.b1, sh.p1);  // the tail pair first
+            rest_end = pstart;
+        } else {
+            seek(p, sh.lo, sh.b0, sh.p0);
         }
     }
-    __device__ bool done() const { return x >= hi; }
+    __device__ bool done() const { return x >= end && rest_end < 0; }
 
     // Fills m for the tile at unit x and advances; returns the tile index
     // within the pair.
@@ -214,7 +249,7 @@ struct TileWalker {
             nseg = c1 - c0 + 1;
             first_slot = (range_lo(c0, W, N) >= pstart) ? 2 * c0 : 2 * c0 + 1;
         }
-        if (x == hi - 1 || t == T - 1) flags |= kLast;
+        if (x == end - 1 || t == T - 1) flags |= kLast;
         if (!valid) flags |= kBad;
         m->b = b; m->g = g; m->key0 = t * kPage; m->leff = leff;
         m->flags = flags; m->slot = slot; m->nseg = nseg; m->first_slot = first_slot;
@@ -226,11 +261,16 @@ struct TileWalker {
             x += kHead;
             if (++g == p.Hkv) {
                 g = 0;
-                if (x < hi) {
+                if (x < end) {
                     ++b;
                     T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
                 }
             }
+        }
+        if (x >= end && rest_end >= 0) {           // the tail pair is done: the rest
+            end = rest_end;
+            rest_end = -1;
+            seek(p, lo, b0, p0);
         }
         return tile;
     }
@@ -249,6 +289,7 @@ struct ProducerSmem {
     int qcopies;           // copies of the query rows per Q buffer
     int qcopy_rows;        // rows between consecutive copies
     int nqbuf;             // Q buffers in the ring (1 or 2)
+    bool tail_first;       // walk a range's split last pair first (TileWalker)
 };
 
 // Meta word layout: meta[2s] = {b, g, key0, leff}; meta[2s+1] = {flags |
@@ -277,7 +318,7 @@ __device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CU
     uint32_t qarmed = 0, qarmed_parity = 0;
     bool ok = true;
     TileWalker wk;
-    wk.init(p, sh);
+    wk.init(p, sh, sm.tail_first);
     while (!wk.done()) {
         if (!mbar_wait(sm.bar_empty + 8 * st, ph ^ 1)) { ok = false; break; }
         TileMeta m;

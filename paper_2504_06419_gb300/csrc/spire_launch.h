@@ -46,8 +46,9 @@ constexpr int stages() {
     constexpr int kp = key_parts(MT);
     constexpr int nw = MT * kp;
     constexpr int qbuf = 2 * (D / 64) * MT * 16 * 128;
-    constexpr int fixed = nw * 16 * (D + 8) * 4 + ((nw * 16 * 8 + 1023) / 1024) * 1024 + qbuf +
-                          8 * 32 + 512 + (2 * 8 + 5) * 8 + 1024;
+    constexpr int fixed = 2 * nw * 8 * (D + 8) * 4 +
+                          ((2 * nw * 8 * 8 + 2 * 32 + 1023) / 1024) * 1024 + qbuf + 8 * 32 + 512 +
+                          (2 * 8 + 9) * 8 + 1024;
     constexpr int stage = 2 * 64 * D * 2;
     constexpr int n = (kMaxDynSmem - fixed) / stage;
     return n > 8 ? 8 : n;

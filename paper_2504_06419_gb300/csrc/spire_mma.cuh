@@ -11,9 +11,15 @@
 //                       It keeps Q in registers for the current pair, runs
 //                       S = Q K^T and O += P V on the tensor cores and an
 //                       fp32 online softmax in base 2.
-// At the end of a pair's segment the KP key slices are merged through shared
-// memory and the result is written to the output, or to a partial slot that
-// the last-arriving CTA merges (see spire_common.cuh).
+//   warp NW+1 (epilogue) at the end of a pair's segment the consumers only
+//                       hand their (O, m, l) rows to one of two shared-memory
+//                       buffers and go on with the next segment; this warp
+//                       merges the KP key slices and writes the result to the
+//                       output, or to a partial slot that the last-arriving
+//                       CTA merges (see spire_common.cuh), publishing with a
+//                       fence and an atomic, off the consumers' path.
+// The kernel serves pairs of at most 8 query rows (one m-tile, rows 8..15 of
+// the MMA are padding), so a buffer holds 8 rows per consumer warp.
 //
 // Precision: P enters the PV product as P_hi + P_lo, two bf16 terms carrying
 // ~16 mantissa bits, so rounding P to bf16 (~1.7e-3 rms relative) never
@@ -27,23 +33,27 @@ namespace spire {
 template <int D, int MT, int KP, int NST>
 struct MmaCfg {
     static constexpr int NW = MT * KP;            // consumer warps
-    static constexpr int THREADS = 32 * (NW + 1); // + one producer warp
+    static constexpr int THREADS = 32 * (NW + 2); // + a producer and an epilogue warp
     static constexpr int KW = kPage / KP;         // keys per consumer warp per tile
     static constexpr int NT = KW / 8;             // S n-tiles per warp
     static constexpr int KK = KW / 16;            // PV k-steps per warp
     static constexpr int TILE = kPage * D * 2;    // bytes of one K (or V) tile
     static constexpr int STAGE = 2 * TILE;
     static constexpr int SCR = D + 8;             // floats per scratch row
-    static constexpr int OFF_SCR_O = NST * STAGE;
-    static constexpr int OFF_SCR_ML = OFF_SCR_O + NW * 16 * SCR * 4;
+    static constexpr int SR = 8;                  // scratch rows per warp (R <= 8)
+    static constexpr int SCR_BUF = NW * SR * SCR; // floats of one hand-over buffer
+    static constexpr int OFF_SCR_O = NST * STAGE;                  // [2][NW][SR][SCR]
+    static constexpr int OFF_SCR_ML = OFF_SCR_O + 2 * SCR_BUF * 4; // [2][NW][SR] float2
+    static constexpr int OFF_SCR_INFO = OFF_SCR_ML + 2 * NW * SR * 8;   // [2] int4 x 2
     static constexpr int QHALF = MT * 16 * 128;         // one 64-column half of a Q buffer
     static constexpr int QBUF = (D / 64) * QHALF;       // Q of one pair (rows padded to MT*16)
-    static constexpr int OFF_Q = ((OFF_SCR_ML + NW * 16 * 8 + 1023) / 1024) * 1024;
+    static constexpr int OFF_Q = ((OFF_SCR_INFO + 2 * 32 + 1023) / 1024) * 1024;
     static constexpr int OFF_META = OFF_Q + 2 * QBUF;
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
     static constexpr int OFF_BAR = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16 + 16;
-    static constexpr int SMEM = OFF_BAR + (2 * NST + 5) * 8 + 1024;  // + alignment slack
+    static constexpr int SMEM = OFF_BAR + (2 * NST + 9) * 8 + 1024;  // + alignment slack
     static_assert(KW >= 16 && NT % 2 == 0, "each warp needs >= 16 keys of a tile");
+    static_assert(MT == 1, "one m-tile: the kernel serves at most 8 query rows");
     static_assert(D % 64 == 0, "head_dim must be a multiple of 64");
     // 128-byte swizzled TMA destinations must sit on 1024-byte boundaries
     static_assert(STAGE % 1024 == 0 && OFF_Q % 1024 == 0 && QHALF % 1024 == 0,
@@ -64,12 +74,13 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     float2* const scr_ml = reinterpret_cast<float2*>(sbase + C::OFF_SCR_ML);
     int4* const meta = reinterpret_cast<int4*>(sbase + C::OFF_META);
     SchedShared* const sh = reinterpret_cast<SchedShared*>(sbase + C::OFF_SCHED);
-    int* const s_flag = reinterpret_cast<int*>(sbase + C::OFF_BAR - 16);
     const uint32_t bar_full = base + C::OFF_BAR;          // NST barriers
     const uint32_t bar_empty = bar_full + NST * 8;         // NST barriers
-    const uint32_t bar_cons = bar_empty + NST * 8;         // consumer-wide barrier
-    const uint32_t bar_qfull = bar_cons + 8;               // 2 barriers: Q buffer landed
+    const uint32_t bar_qfull = bar_empty + NST * 8;        // 2 barriers: Q buffer landed
     const uint32_t bar_qempty = bar_qfull + 16;            // 2 barriers: Q buffer read
+    const uint32_t bar_sfull = bar_qempty + 16;            // 2: a hand-over buffer was filled
+    const uint32_t bar_sempty = bar_sfull + 16;            // 2: the epilogue is done with it
+    int4* const scr_info = reinterpret_cast<int4*>(sbase + C::OFF_SCR_INFO);
     const uint32_t qsm = base + C::OFF_Q;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -78,10 +89,11 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
             mbar_init(bar_full + 8 * s, 1);
             mbar_init(bar_empty + 8 * s, C::NW);
         }
-        mbar_init(bar_cons, 32 * C::NW);
         for (int b = 0; b < 2; ++b) {
             mbar_init(bar_qfull + 8 * b, 1);
             mbar_init(bar_qempty + 8 * b, C::NW);
+            mbar_init(bar_sfull + 8 * b, C::NW);
+            mbar_init(bar_sempty + 8 * b, 1);
         }
         fence_barrier_init();
         if (blockIdx.x == 0) p.header[0] = gridDim.x;
@@ -99,10 +111,87 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         // ------------------------------------------------------ producer
         if (lane != 0) return;
         const ProducerSmem psm{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
-                               bar_empty, bar_qfull, bar_qempty, 1, 0, 2};
+                               bar_empty, bar_qfull, bar_qempty, 1, 0, 2, true};
         const uint32_t err = produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, psm);
         if (err) atomicOr(&p.err[blockIdx.x], (int)err);
         return;
+    }
+    if (warp == C::NW + 1) {
+        // ------------------------------------------------------ epilogue
+        const float NEG_INF = __int_as_float(0xff800000);
+        const float NANF = __int_as_float(0x7fc00000);
+        constexpr int D4 = D / 4;
+        for (uint32_t n = 0;; ++n) {
+            const int sb = n & 1;
+            if (!mbar_wait(bar_sfull + 8 * sb, (n >> 1) & 1)) {
+                if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
+                return;
+            }
+            const int4 i0 = scr_info[2 * sb], i1 = scr_info[2 * sb + 1];
+            if (i1.y) return;                          // the consumers have finished
+            const int cb = i0.x, cg = i0.y, cslot = i0.z, cnseg = i0.w, cfirst = i1.x;
+            const float* so = scr_o + sb * C::SCR_BUF;
+            const float2* sml = scr_ml + sb * C::NW * C::SR;
+            for (int idx = lane; idx < p.R * D4; idx += 32) {
+                const int r = idx / D4, d4 = idx - r * D4;
+                float M = NEG_INF;
+                bool nan = false;
+#pragma unroll
+                for (int kq = 0; kq < KP; ++kq) {
+                    const float mk = sml[kq * C::SR + r].x;
+                    nan |= (mk != mk);
+                    M = fmaxf(M, mk);
+                }
+                const float Mr = (M == NEG_INF) ? 0.f : M;
+                float lsum = 0.f;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int kq = 0; kq < KP; ++kq) {
+                    const float2 ml = sml[kq * C::SR + r];
+                    const float wgt = ex2(ml.x - Mr);
+                    lsum += wgt * ml.y;
+                    const float4 ov =
+                        *reinterpret_cast<const float4*>(so + (kq * C::SR + r) * C::SCR + 4 * d4);
+                    acc.x += wgt * ov.x; acc.y += wgt * ov.y;
+                    acc.z += wgt * ov.z; acc.w += wgt * ov.w;
+                }
+                float4 res;
+                float lse;
+                if (nan) {
+                    res = make_float4(NANF, NANF, NANF, NANF);
+                    lse = NANF;
+                } else if (lsum > 0.f) {
+                    const float inv = 1.f / lsum;
+                    res = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+                    lse = M + __log2f(lsum);
+                } else {  // no key of this segment is visible to this row
+                    res = make_float4(0.f, 0.f, 0.f, 0.f);
+                    lse = NEG_INF;
+                }
+                if (cnseg == 1) {
+                    *reinterpret_cast<float4*>(out_row(p, cb, cg, r, D) + 4 * d4) = res;
+                } else {
+                    const long long row = (long long)cslot * p.R + r;
+                    *reinterpret_cast<float4*>(p.part_o + row * D + 4 * d4) = res;
+                    if (d4 == 0) p.part_lse[row] = lse;
+                }
+            }
+            __syncwarp();
+            // the buffer is read: the consumers may fill it again
+            if (lane == 0) mbar_arrive(bar_sempty + 8 * sb);
+            if (cnseg > 1) {
+                // publish this segment; the CTA completing the pair merges it
+                __threadfence();
+                __syncwarp();
+                int last = 0;
+                if (lane == 0) last = atomicAdd(p.cnt + cb * p.Hkv + cg, 1) == cnseg - 1;
+                last = __shfl_sync(0xffffffffu, last, 0);
+                if (last) {
+                    __threadfence();
+                    merge_pair<D>(p, cb, cg, cnseg, cfirst, lane, 32);
+                }
+            }
+        }
     }
 
     // ---------------------------------------------------------- consumers
@@ -110,7 +199,6 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     const int gq = lane >> 2, tq = lane & 3;          // mma group / thread-in-group
     const int r0 = mt * 16 + gq, r1 = r0 + 8;         // the two rows this thread holds
     const int wkey = kp * C::KW;                      // first key of this warp in a tile
-    const int ctid = threadIdx.x;                     // 0 .. 32*NW-1
     const float sl2 = p.sl2;
     const float NEG_INF = __int_as_float(0xff800000);
     const float NANF = __int_as_float(0x7fc00000);
@@ -121,14 +209,31 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     bool poison = false;
     int cur_b = 0, cur_g = 0, cur_slot = 0, cur_nseg = 1, cur_first = 0;
     int lim0 = 0, lim1 = 0, leff = 0;
-    uint32_t st = 0, ph = 0, cph = 0;                 // stage ring / consumer-barrier phase
+    uint32_t st = 0, ph = 0, n_seg = 0;               // stage ring / segments handed over
     uint32_t cq[2] = {0u, 0u};                        // parity of each Q buffer
 
-    auto cbar = [&]() -> bool {                       // all consumer threads
-        mbar_arrive(bar_cons);
-        const bool r = mbar_wait(bar_cons, cph & 1);
-        ++cph;
-        return r;
+    // hand the segment's (O, m, l) rows, or the end of the work, to the epilogue
+    // warp through buffer n_seg & 1 (rows r0 = gq < 8 only: rows 8..15 are padding)
+    auto hand_over = [&](bool term, float lt0) -> bool {
+        const int sb = n_seg & 1;
+        if (!mbar_wait(bar_sempty + 8 * sb, ((n_seg >> 1) & 1) ^ 1)) return false;
+        if (!term) {
+            float* so = scr_o + sb * C::SCR_BUF + (warp * C::SR + gq) * C::SCR;
+#pragma unroll
+            for (int j = 0; j < D / 8; ++j)
+                *reinterpret_cast<float2*>(so + 8 * j + 2 * tq) = make_float2(o[j][0], o[j][1]);
+            if (tq == 0)
+                scr_ml[sb * C::NW * C::SR + warp * C::SR + gq] =
+                    make_float2(poison ? NANF : m0, lt0);
+        }
+        if (warp == 0 && lane == 0) {
+            scr_info[2 * sb] = make_int4(cur_b, cur_g, cur_slot, cur_nseg);
+            scr_info[2 * sb + 1] = make_int4(cur_first, term ? 1 : 0, 0, 0);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_sfull + 8 * sb);
+        ++n_seg;
+        return true;
     };
 
     for (;;) {
@@ -138,7 +243,10 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         }
         const int4 ma = meta[2 * st], mb = meta[2 * st + 1];
         const int flags = mb.x & 0xff;
-        if (flags & kTerm) return;
+        if (flags & kTerm) {
+            if (!hand_over(true, 0.f) && lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
+            return;
+        }
         if (flags & kFirst) {
             const int flags_q = mb.x;
             cur_b = ma.x; cur_g = ma.y; leff = ma.w;
@@ -286,90 +394,10 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         if (lane == 0) mbar_arrive(bar_empty + 8 * st);
 
         if (flags & kLast) {
-            // ---- segment end: merge the KP key slices of each m-tile
+            // ---- segment end: the row sums over the quad, then hand over
             float lt0 = l0 + __shfl_xor_sync(0xffffffffu, l0, 1);
             lt0 += __shfl_xor_sync(0xffffffffu, lt0, 2);
-            float lt1 = l1 + __shfl_xor_sync(0xffffffffu, l1, 1);
-            lt1 += __shfl_xor_sync(0xffffffffu, lt1, 2);
-            bool ok = cbar();                          // previous readers of the scratch are done
-            float* so = scr_o + warp * 16 * C::SCR;
-#pragma unroll
-            for (int j = 0; j < D / 8; ++j) {
-                *reinterpret_cast<float2*>(so + gq * C::SCR + 8 * j + 2 * tq) =
-                    make_float2(o[j][0], o[j][1]);
-                *reinterpret_cast<float2*>(so + (gq + 8) * C::SCR + 8 * j + 2 * tq) =
-                    make_float2(o[j][2], o[j][3]);
-            }
-            if (tq == 0) {
-                scr_ml[warp * 16 + gq] = make_float2(poison ? NANF : m0, lt0);
-                scr_ml[warp * 16 + gq + 8] = make_float2(poison ? NANF : m1, lt1);
-            }
-            ok = ok && cbar();
-            constexpr int D4 = D / 4;
-            for (int idx = ctid; ok && idx < MT * 16 * D4; idx += 32 * C::NW) {
-                const int mtm = idx / (16 * D4);
-                const int rem = idx - mtm * 16 * D4;
-                const int rl = rem / D4, d4 = rem - rl * D4;
-                const int r = mtm * 16 + rl;
-                if (r >= p.R) continue;
-                float M = NEG_INF;
-                bool nan = false;
-#pragma unroll
-                for (int kq = 0; kq < KP; ++kq) {
-                    const float mk = scr_ml[(mtm * KP + kq) * 16 + rl].x;
-                    nan |= (mk != mk);
-                    M = fmaxf(M, mk);
-                }
-                const float Mr = (M == NEG_INF) ? 0.f : M;
-                float lsum = 0.f;
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-                for (int kq = 0; kq < KP; ++kq) {
-                    const int w2 = mtm * KP + kq;
-                    const float2 ml = scr_ml[w2 * 16 + rl];
-                    const float wgt = ex2(ml.x - Mr);
-                    lsum += wgt * ml.y;
-                    const float4 ov =
-                        *reinterpret_cast<const float4*>(scr_o + (w2 * 16 + rl) * C::SCR + 4 * d4);
-                    acc.x += wgt * ov.x; acc.y += wgt * ov.y;
-                    acc.z += wgt * ov.z; acc.w += wgt * ov.w;
-                }
-                float4 res;
-                float lse;
-                if (nan) {
-                    res = make_float4(NANF, NANF, NANF, NANF);
-                    lse = NANF;
-                } else if (lsum > 0.f) {
-                    const float inv = 1.f / lsum;
-                    res = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-                    lse = M + __log2f(lsum);
-                } else {  // no key of this segment is visible to this row
-                    res = make_float4(0.f, 0.f, 0.f, 0.f);
-                    lse = NEG_INF;
-                }
-                if (cur_nseg == 1) {
-                    *reinterpret_cast<float4*>(out_row(p, cur_b, cur_g, r, D) + 4 * d4) = res;
-                } else {
-                    const long long row = (long long)cur_slot * p.R + r;
-                    *reinterpret_cast<float4*>(p.part_o + row * D + 4 * d4) = res;
-                    if (d4 == 0) p.part_lse[row] = lse;
-                }
-            }
-            if (ok && cur_nseg > 1) {
-                // publish this segment; the CTA completing the pair merges it
-                __threadfence();
-                ok = cbar();
-                if (ctid == 0) {
-                    const int old = atomicAdd(p.cnt + cur_b * p.Hkv + cur_g, 1);
-                    *s_flag = (old == cur_nseg - 1);
-                }
-                ok = ok && cbar();
-                if (ok && *s_flag) {
-                    __threadfence();
-                    merge_pair<D>(p, cur_b, cur_g, cur_nseg, cur_first, ctid, 32 * C::NW);
-                }
-            }
-            if (!ok) {
+            if (!hand_over(false, lt0)) {
                 if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
                 return;
             }

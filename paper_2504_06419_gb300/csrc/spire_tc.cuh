@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(224, 1)
         // ------------------------------------------------------ producer
         if (lane == 0) {
             const ProducerSmem ps{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
-                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC, 1};
+                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC, 1, false};
             err |= produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
         }
     } else if (warp == 1) {
