@@ -172,16 +172,20 @@ __global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n)
 // ------------------------------------------------------------- MagicDec gather
 // MagicDec's draft attends, with positions inside the reduced cache, to the
 // sink + window entries of the target's own paged cache (Section 3.1
-// footnote).  This kernel builds that reduced cache: one warp per row.
-//   sequence rows  n_vis[b] = number of visible entries (0 if t is out of
-//                  range or a visible page id is outside the cache)
-//   K / V rows     entry c of (b, g): the text position p, K turned by
-//                  (c - p) (rotary pairs (d, d + D/2)) and rounded to bf16,
-//                  V copied
-//   query rows     q turned by the query's cache index n_vis - 1
-// Angles: (c - p) * freq[d] and its reduction modulo 2 pi in double, sine and
-// cosine of the reduced angle in fp32 (positions up to 2^31 keep their
-// accuracy).
+// footnote).  This kernel builds that reduced cache, one warp per item:
+//   sequence items  n_vis[b] = number of visible entries (0 if t is out of
+//                   range or a visible page id is outside the cache)
+//   row items       1/32 of the slots of (b, g): entry c at text position
+//                   p, K turned by (c - p) and rounded to bf16, V copied.  A
+//                   sink keeps its position (c = p) and every window entry
+//                   moves by the same s - w0, so a warp computes its lanes'
+//                   sine and cosine once and applies them to all its rows
+//   query items     q turned by the query's cache index n_vis - 1
+// Angles: the product with the frequency and its reduction modulo 2 pi in
+// double, sine and cosine of the reduced angle in fp32 (positions up to 2^31
+// keep their accuracy).
+constexpr int kMdParts = 32;          // row items per (sequence, KV head): few rows each
+
 struct MdParams {
     const __nv_bfloat16* q;        // [B, Hq, D], not rotated
     const __nv_bfloat16* k_cache;  // [num_pages, Hkv, 64, D], keys turned by text position
@@ -208,40 +212,43 @@ __device__ __forceinline__ MdVisible md_visible(const MdParams& p, int t) {
     return v;
 }
 
-// turn pairs (d, d + D/2) of a row by delta positions (lane handles d = lane + 32 i)
-__device__ __forceinline__ void md_rotate_row(const __nv_bfloat16* src, __nv_bfloat16* dst,
-                                              long long delta, const MdParams& p, int lane) {
-    const int half = p.D / 2;
+// sine and cosine of delta * freq[d] (delta != 0, rotation on)
+__device__ __forceinline__ void md_sincos(const MdParams& p, long long delta, int d, float* sn,
+                                          float* cs) {
     const double kTwoPi = 6.283185307179586476925286766559;
     const double kInvTwoPi = 0.15915494309189533576888376337251;
-    for (int d = lane; d < half; d += 32) {
+    const double ang = (double)delta * p.freq[d];
+    sincosf((float)fma(-kTwoPi, rint(ang * kInvTwoPi), ang), sn, cs);
+}
+
+// turn the pairs (d, d + D/2) of a row, lane handling d = lane + 32 i, by the
+// angles given as sines / cosines per i (identity: sn = 0, cs = 1), bf16 out
+__device__ __forceinline__ void md_turn_row(const __nv_bfloat16* src, __nv_bfloat16* dst,
+                                            const float* sn, const float* cs, int half,
+                                            int lane) {
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int d = lane + 32 * i;
+        if (d >= half) break;
         const float a0 = __bfloat162float(src[d]), a1 = __bfloat162float(src[d + half]);
-        float r0 = a0, r1 = a1;
-        if (p.rotate && delta != 0) {
-            const double ang = (double)delta * p.freq[d];
-            const double red = fma(-kTwoPi, rint(ang * kInvTwoPi), ang);
-            float sn, cs;
-            sincosf((float)red, &sn, &cs);
-            r0 = a0 * cs - a1 * sn;
-            r1 = a1 * cs + a0 * sn;
-        }
-        dst[d] = __float2bfloat16_rn(r0);
-        dst[d + half] = __float2bfloat16_rn(r1);
+        dst[d] = __float2bfloat16_rn(a0 * cs[i] - a1 * sn[i]);
+        dst[d + half] = __float2bfloat16_rn(a1 * cs[i] + a0 * sn[i]);
     }
 }
 
 __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) {
-    const int lane = threadIdx.x & 31;
-    const long long n_kv = (long long)p.B * p.Hkv * p.S;
-    const long long total = p.B + n_kv + (long long)p.B * p.Hq;
+    const int lane = threadIdx.x & 31, half = p.D / 2;
+    const long long n_rows = (long long)p.B * p.Hkv * kMdParts;
+    const long long total = p.B + n_rows + (long long)p.B * p.Hq;
+    const int rpp = (p.S + kMdParts - 1) / kMdParts;         // slots per row item
     for (long long item = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5; item < total;
          item += ((long long)gridDim.x * blockDim.x) >> 5) {
         if (item < p.B) {
-            // sequence row: the visible count, after checking every visible page
+            // sequence item: the visible count, after checking every visible page
             const int b = (int)item;
-            MdVisible v = md_visible(p, p.ctx_lens[b]);
-            bool ok = v.n > 0;
             const int t = p.ctx_lens[b];
+            const MdVisible v = md_visible(p, t);
+            bool ok = v.n > 0;
             const int pg_s = v.s > 0 ? (v.s - 1) / kPage + 1 : 0;     // pages of the sinks
             const int pg_w0 = v.w0 / kPage, pg_w1 = ok ? (t - 1) / kPage : -1;
             for (int pg = lane; ok && pg < pg_s; pg += 32) {
@@ -254,29 +261,47 @@ __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) 
             }
             ok = __all_sync(0xffffffffu, ok);
             if (lane == 0) p.n_vis[b] = ok ? v.n : 0;
-        } else if (item < p.B + n_kv) {
+        } else if (item < p.B + n_rows) {
             long long r = item - p.B;
-            const int c = (int)(r % p.S); r /= p.S;
+            const int part = (int)(r % kMdParts); r /= kMdParts;
             const int g = (int)(r % p.Hkv);
             const int b = (int)(r / p.Hkv);
             const MdVisible v = md_visible(p, p.ctx_lens[b]);
-            if (c >= v.n) continue;
-            const int pos = c < v.s ? c : v.w0 + (c - v.s);
-            const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
-            if (id < 0 || id >= p.num_pages) continue;   // the sequence row reports it
-            const long long src = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * p.D;
-            const long long dk = ((((long long)b * 2 + 0) * p.Hkv + g) * p.S + c) * p.D;
-            const long long dv = ((((long long)b * 2 + 1) * p.Hkv + g) * p.S + c) * p.D;
-            md_rotate_row(p.k_cache + src, p.kv + dk, (long long)c - pos, p, lane);
-            for (int d = 2 * lane; d < p.D; d += 64)
-                *reinterpret_cast<__nv_bfloat162*>(p.kv + dv + d) =
-                    *reinterpret_cast<const __nv_bfloat162*>(p.v_cache + src + d);
+            const int c0 = part * rpp, c1 = min(v.n, c0 + rpp);
+            if (c0 >= c1) continue;
+            // the window's common turn s - w0, once per lane
+            float wsn[2] = {0.f, 0.f}, wcs[2] = {1.f, 1.f};
+            const float zsn[2] = {0.f, 0.f}, ocs[2] = {1.f, 1.f};
+            if (p.rotate && v.s != v.w0)
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+                    if (lane + 32 * i < half) md_sincos(p, (long long)v.s - v.w0, lane + 32 * i, &wsn[i], &wcs[i]);
+#pragma unroll 2
+            for (int c = c0; c < c1; ++c) {
+                const bool sink = c < v.s;
+                const int pos = sink ? c : v.w0 + (c - v.s);
+                const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
+                if (id < 0 || id >= p.num_pages) continue;   // the sequence item reports it
+                const long long src = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * p.D;
+                const long long dk = ((((long long)b * 2 + 0) * p.Hkv + g) * p.S + c) * p.D;
+                const long long dv = ((((long long)b * 2 + 1) * p.Hkv + g) * p.S + c) * p.D;
+                md_turn_row(p.k_cache + src, p.kv + dk, sink ? zsn : wsn, sink ? ocs : wcs, half,
+                            lane);
+                for (int d = 2 * lane; d < p.D; d += 64)
+                    *reinterpret_cast<__nv_bfloat162*>(p.kv + dv + d) =
+                        *reinterpret_cast<const __nv_bfloat162*>(p.v_cache + src + d);
+            }
         } else {
-            const long long r = item - p.B - n_kv;
+            const long long r = item - p.B - n_rows;
             const int b = (int)(r / p.Hq);
             const MdVisible v = md_visible(p, p.ctx_lens[b]);
             if (v.n == 0) continue;
-            md_rotate_row(p.q + r * p.D, p.q_eff + r * p.D, v.n - 1, p, lane);
+            float sn[2] = {0.f, 0.f}, cs[2] = {1.f, 1.f};
+            if (p.rotate && v.n > 1)
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+                    if (lane + 32 * i < half) md_sincos(p, v.n - 1, lane + 32 * i, &sn[i], &cs[i]);
+            md_turn_row(p.q + r * p.D, p.q_eff + r * p.D, sn, cs, half, lane);
         }
     }
 }
@@ -497,7 +522,7 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
     // the rotary frequencies theta^(-2d/D): per-call constants, in double
     for (int d = 0; d < desc->head_dim / 2; ++d)
         mp.freq[d] = mp.rotate ? std::pow((double)rope_theta, -2.0 * d / desc->head_dim) : 0.0;
-    const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * S + mp.Hq);
+    const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * kMdParts + mp.Hq);
     long long blocks = (items * 32 + 255) / 256;
     if (blocks > 32LL * di.sms) blocks = 32LL * di.sms;
     magicdec_gather_kernel<<<(unsigned)blocks, 256, 0, s>>>(mp);
