@@ -658,7 +658,7 @@ def spire_arm(args, cfg):
                        "us": app_ms * 1e3, "algorithmic_bytes": ab,
                        "gbs": ab / (app_ms * 1e-3) / 1e9,
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
-                       "launches": 3},
+                       "launches": 1},
                    "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
                    "magicdec_draft_step": {
                        "what": "spire_magicdec_attention: sink %d + window %d over the target's "

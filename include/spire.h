@@ -232,9 +232,8 @@ typedef struct spire_append_desc {
 
 /*
  * spire_feedback_append_workspace_bytes -- workspace size for
- * spire_feedback_append (the memory vectors as two bf16 parts, split-K
- * partials, rotary frequencies and the device error word).
- * Returns 0 for invalid arguments.
+ * spire_feedback_append (the device error words; the same 2304 bytes for
+ * every valid descriptor).  Returns 0 for invalid arguments.
  */
 SPIRE_API size_t spire_feedback_append_workspace_bytes(const spire_append_desc *desc);
 
@@ -256,9 +255,12 @@ SPIRE_API size_t spire_feedback_append_workspace_bytes(const spire_append_desc *
  *            cache is the [B, 2, Hkv, S, D] block spire_draft_sparse_attention
  *            reads), updated in place; no other slot is written.
  *   workspace >= spire_feedback_append_workspace_bytes(desc) bytes.
- * The product runs on the tensor cores with the memory vector split into two
- * bf16 parts (about 16 significant bits) and fp32 accumulation, so an entry is
- * within one bf16 unit of the exactly rounded value.  A sequence with
+ * The projection is linear, so the kernel computes sum_l a_l (W x_l) with
+ * a = softmax(mix_w[i, :]): exact bf16 products accumulated in fp32 on the
+ * tensor cores, the accumulators mixed in fp32; an entry is within one bf16
+ * unit of the exactly rounded value up to the fp32 accumulation error.  One
+ * launch (thread-block clusters, programmatic dependent launch; a one-thread
+ * error-word clear before it only for grids above 512 CTAs).  A sequence with
  * pos[b] < 0 is not written and sets SPIRE_DEVERR_CTX_LEN.  Pointers x, w_kv
  * and kv must be 16-byte aligned, the workspace 256-byte aligned.
  */

@@ -160,6 +160,35 @@ bool encode_2d_bf16_map(CUtensorMap* map, const void* base, uint64_t inner, uint
     return r == CUDA_SUCCESS;
 }
 
+uint64_t rope_turn_fixed(double freq) {
+    // 1 / (2 pi) = kInv2PiHi + kInv2PiLo to about 2^-107; freq / (2 pi) =
+    // ph + pe with ph = fl(freq * hi) and pe its error plus freq * lo
+    const double kInv2PiHi = 0.15915494309189535;
+    const double kInv2PiLo = -9.839338337591243e-18;
+    if (!(freq > 0.0)) return 0;
+    const double ph = freq * kInv2PiHi;
+    const double pe = std::fma(freq, kInv2PiHi, -ph) + freq * kInv2PiLo;
+    const double two64 = 18446744073709551616.0;
+    // ph * 2^64 < 2^62 truncates to an integer with an error below one unit
+    // (none once it exceeds 2^53); pe * 2^64 adds the rest, rounded
+    const double hi = std::floor(ph * two64);
+    return (uint64_t)hi + (uint64_t)(int64_t)std::llround(ph * two64 - hi + pe * two64);
+}
+
+bool encode_3d_bf16_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t mid,
+                        uint64_t outer, uint32_t box_inner, uint32_t box_mid, uint32_t box_outer) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {inner, mid, outer};
+    cuuint64_t strides[2] = {inner * 2, inner * 2 * mid};
+    cuuint32_t box[3] = {box_inner, box_mid, box_outer};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 namespace {
 
 // Zeroes the per-pair arrival counters; lets the attention kernel launched
@@ -181,9 +210,9 @@ __global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n)
 //                   moves by the same s - w0, so a warp computes its lanes'
 //                   sine and cosine once and applies them to all its rows
 //   query items     q turned by the query's cache index n_vis - 1
-// Angles: the product with the frequency and its reduction modulo 2 pi in
-// double, sine and cosine of the reduced angle in fp32 (positions up to 2^31
-// keep their accuracy).
+// Angles: reduced modulo 2 pi exactly in 64-bit fixed point (rope_sincos),
+// sine and cosine of the reduced angle in fp32 (positions up to 2^31 keep
+// their accuracy).
 constexpr int kMdParts = 32;          // row items per (sequence, KV head): few rows each
 
 struct MdParams {
@@ -196,7 +225,7 @@ struct MdParams {
     __nv_bfloat16* q_eff;          // [B, Hq, D]
     int32_t* n_vis;                // [B]
     int B, Hq, Hkv, D, S, n_sink, window, max_pages, num_pages, rotate;
-    double freq[64];
+    uint64_t fturn[64];            // theta^(-2d/D) / (2 pi) as 64-bit fractions
 };
 
 struct MdVisible {
@@ -212,13 +241,12 @@ __device__ __forceinline__ MdVisible md_visible(const MdParams& p, int t) {
     return v;
 }
 
-// sine and cosine of delta * freq[d] (delta != 0, rotation on)
-__device__ __forceinline__ void md_sincos(const MdParams& p, long long delta, int d, float* sn,
+// sine and cosine of delta * freq[d] (delta != 0, rotation on); the turn
+// constants come from shared memory (lanes index them: from kernel
+// parameters the reads would serialise)
+__device__ __forceinline__ void md_sincos(const uint64_t* turn, long long delta, int d, float* sn,
                                           float* cs) {
-    const double kTwoPi = 6.283185307179586476925286766559;
-    const double kInvTwoPi = 0.15915494309189533576888376337251;
-    const double ang = (double)delta * p.freq[d];
-    sincosf((float)fma(-kTwoPi, rint(ang * kInvTwoPi), ang), sn, cs);
+    rope_sincos(delta, turn[d], sn, cs);
 }
 
 // turn the pairs (d, d + D/2) of a row, lane handling d = lane + 32 i, by the
@@ -237,6 +265,9 @@ __device__ __forceinline__ void md_turn_row(const __nv_bfloat16* src, __nv_bfloa
 }
 
 __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) {
+    __shared__ uint64_t turn[64];
+    if (threadIdx.x < 64) turn[threadIdx.x] = p.fturn[threadIdx.x];
+    __syncthreads();
     const int lane = threadIdx.x & 31, half = p.D / 2;
     const long long n_rows = (long long)p.B * p.Hkv * kMdParts;
     const long long total = p.B + n_rows + (long long)p.B * p.Hq;
@@ -275,7 +306,7 @@ __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) 
             if (p.rotate && v.s != v.w0)
 #pragma unroll
                 for (int i = 0; i < 2; ++i)
-                    if (lane + 32 * i < half) md_sincos(p, (long long)v.s - v.w0, lane + 32 * i, &wsn[i], &wcs[i]);
+                    if (lane + 32 * i < half) md_sincos(turn, (long long)v.s - v.w0, lane + 32 * i, &wsn[i], &wcs[i]);
 #pragma unroll 2
             for (int c = c0; c < c1; ++c) {
                 const bool sink = c < v.s;
@@ -300,7 +331,7 @@ __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) 
             if (p.rotate && v.n > 1)
 #pragma unroll
                 for (int i = 0; i < 2; ++i)
-                    if (lane + 32 * i < half) md_sincos(p, v.n - 1, lane + 32 * i, &sn[i], &cs[i]);
+                    if (lane + 32 * i < half) md_sincos(turn, v.n - 1, lane + 32 * i, &sn[i], &cs[i]);
             md_turn_row(p.q + r * p.D, p.q_eff + r * p.D, sn, cs, half, lane);
         }
     }
@@ -519,9 +550,12 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
     mp.max_pages = desc->max_pages_per_seq;
     mp.num_pages = desc->num_pages;
     mp.rotate = rope_theta > 0.f;
-    // the rotary frequencies theta^(-2d/D): per-call constants, in double
+    // the rotary frequencies theta^(-2d/D) (the same libm pow as the
+    // definition) as per-call fixed-point turn constants
     for (int d = 0; d < desc->head_dim / 2; ++d)
-        mp.freq[d] = mp.rotate ? std::pow((double)rope_theta, -2.0 * d / desc->head_dim) : 0.0;
+        mp.fturn[d] = mp.rotate
+                          ? rope_turn_fixed(std::pow((double)rope_theta, -2.0 * d / desc->head_dim))
+                          : 0;
     const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * kMdParts + mp.Hq);
     long long blocks = (items * 32 + 255) / 256;
     if (blocks > 32LL * di.sms) blocks = 32LL * di.sms;
@@ -543,15 +577,20 @@ int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {
 spire_status spire_get_device_error(const void* workspace, int32_t* code_out, void* stream) {
     if (!workspace || !code_out) return SPIRE_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // the header and the per-CTA words are contiguous: one copy
-    int32_t buf[(kHeaderBytes + kMaxCtas * 4) / 4];
-    if (cudaMemcpyAsync(buf, workspace, sizeof(buf), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    // the header word first, then exactly the words it counts: a workspace
+    // holds at least kHeaderBytes plus the words its last call wrote
+    int32_t n = 0;
+    if (cudaMemcpyAsync(&n, workspace, sizeof(n), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
         return SPIRE_ERR_CUDA;
-    if (cudaStreamSynchronize(s) != cudaSuccess) return SPIRE_ERR_CUDA;
-    int n = buf[0];
-    if (n < 0 || n > kMaxCtas) n = kMaxCtas;
+    if (n < 0 || n > kMaxCtas) n = 0;
+    int32_t buf[kMaxCtas];
+    if (n > 0 && (cudaMemcpyAsync(buf, static_cast<const char*>(workspace) + kHeaderBytes,
+                                  (size_t)n * 4, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+                  cudaStreamSynchronize(s) != cudaSuccess))
+        return SPIRE_ERR_CUDA;
     int32_t v = 0;
-    for (int c = 0; c < n; ++c) v |= buf[kHeaderBytes / 4 + c];
+    for (int c = 0; c < n; ++c) v |= buf[c];
     *code_out = v;
     return SPIRE_OK;
 }

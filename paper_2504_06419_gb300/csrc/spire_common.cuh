@@ -43,6 +43,22 @@ constexpr uint32_t kErrTimeout = 4u;
 
 enum Mode : int32_t { kModeVerify = 0, kModeDraft = 1 };
 
+// Sine and cosine of the rotary angle delta * freq for |delta| < 2^31, from
+// fturn = freq / (2 pi) as a 64-bit binary fraction (the host's
+// rope_turn_fixed): delta * fturn modulo 2^64 is the angle in turns modulo
+// one, exact in integer arithmetic; its top 32 bits, read as a signed
+// fraction of a turn, give the reduced angle in [-pi, pi) in fp32 (about
+// 2e-7 rad of rounding), whose sine and cosine come from the hardware
+// approximation (absolute error about 2^-21 on [-pi, pi]; the rotated values
+// are rounded to bf16, 2^-9 relative).  No double arithmetic on the device:
+// GB300's double-precision rate is a small fraction of its fp32 rate.
+__device__ __forceinline__ void rope_sincos(long long delta, uint64_t fturn, float* sn,
+                                            float* cs) {
+    const uint64_t t = (uint64_t)delta * fturn;
+    const float a = (float)(int32_t)(uint32_t)(t >> 32) * 1.4629180792671596e-9f;  // 2 pi / 2^32
+    __sincosf(a, sn, cs);
+}
+
 // Stage flags passed from the producer to the consumers.
 enum : int32_t { kFirst = 1, kLast = 2, kBad = 4, kTerm = 8 };
 

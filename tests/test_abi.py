@@ -133,17 +133,13 @@ def _adesc(spire, **kw):
 
 
 def test_append_workspace_depends_only_on_shapes(spire):
-    def expect(B, n_dl, d_model, F, splits):
-        m = (2 * n_dl * B * d_model * 2 + 255) // 256 * 256     # m_hi and m_lo, bf16
-        return 512 + 512 + m + splits * n_dl * B * F * 4         # header, frequencies, partials
+    # the header word and one device error word per CTA (at most 512): the
+    # kernel keeps its split partials in shared memory, so no shape needs more
     d = _adesc(spire)
-    n = spire.spire_feedback_append_workspace_bytes(d)
-    # 2 layers x 16 row blocks x 1 token block = 32 tiles: up to 8 K splits
-    assert n == expect(64, 2, 4096, 2048, 8)
-    # 3 token blocks of 128: 96 tiles, up to 2 splits
-    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, batch=300)) == \
-        expect(300, 2, 4096, 2048, 2)
-    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire)) == n
+    n = 256 + 4 * 512
+    assert spire.spire_feedback_append_workspace_bytes(d) == n
+    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, batch=300)) == n
+    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, num_act=16, d_model=64)) == n
 
 
 @pytest.mark.parametrize("kw", [
