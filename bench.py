@@ -448,17 +448,40 @@ def spire_arm(args, cfg):
            sum(x.numel() * 2 for x in h_dq) + sum(x.numel() * 4 for x in h_dctx))
     d2h = h_out.numel() * 4 + sum(x.numel() * 4 for x in h_dout)
 
+    # Within a step the uploads run on their own stream ahead of the kernels
+    # that need them and each result goes back on another while the next
+    # kernels run, as a serving loop overlaps them; nothing crosses a step.
+    up, down = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev = lambda: torch.cuda.Event()
+
     def e2e_step():
-        d_q.copy_(h_q, non_blocking=True)
-        d_ctx.copy_(h_ctx, non_blocking=True)
-        d_bt.copy_(h_bt, non_blocking=True)
+        t0, ins, outs, done = ev(), [ev() for _ in range(k + 1)], [ev() for _ in range(k + 1)], ev()
+        t0.record(stream)
+        up.wait_event(t0)
+        with torch.cuda.stream(up):
+            d_q.copy_(h_q, non_blocking=True)
+            d_ctx.copy_(h_ctx, non_blocking=True)
+            d_bt.copy_(h_bt, non_blocking=True)
+            ins[0].record(up)
+            for j in range(k):
+                d_dq[j].copy_(h_dq[j], non_blocking=True)
+                d_dctx[j].copy_(h_dctx[j], non_blocking=True)
+                ins[j + 1].record(up)
+        stream.wait_event(ins[0])
         call_verify(q=d_q, ctx=d_ctx, bt=d_bt, out=out_v)
-        h_out.copy_(out_v, non_blocking=True)
+        outs[0].record(stream)
         for j in range(k):
-            d_dq[j].copy_(h_dq[j], non_blocking=True)
-            d_dctx[j].copy_(h_dctx[j], non_blocking=True)
+            stream.wait_event(ins[j + 1])
             call_draft(j, q=d_dq[j], ctx=d_dctx[j], out=out_d[j])
-            h_dout[j].copy_(out_d[j], non_blocking=True)
+            outs[j + 1].record(stream)
+        with torch.cuda.stream(down):
+            down.wait_event(outs[0])
+            h_out.copy_(out_v, non_blocking=True)
+            for j in range(k):
+                down.wait_event(outs[j + 1])
+                h_dout[j].copy_(out_d[j], non_blocking=True)
+            done.record(down)
+        stream.wait_event(done)
 
     for _ in range(max(3, args.warmup)):
         e2e_step()
