@@ -631,6 +631,58 @@ def spire_arm(args, cfg):
                                            Hkv, D) for j in range(k))
     del md_ws
 
+    # ---- draft sweep: B = 512, t log-uniform in [4096, 262144], sink 16, windows 256 /
+    # 1024 / 4096 (bounded caches of 0.57 / 2.2 / 8.6 GB); k steps on one cache per
+    # window (step j sees t + j entries); draft tokens/s = B k / sum of the step times
+    sw_cfg = wl.CONFIGS["draft_sweep"]
+    sw_L = wl.sample_ctx_lens(sw_cfg)
+    sw_k, sw_B = sw_cfg.k, int(sw_L.size)
+    sweep = []
+    for w in sw_cfg.windows:
+        sw_S = sw_cfg.n_sink + w
+        sdi = wl.make_draft(wl.draft_ctx_for_step(sw_L, sw_k, 0), Hq, Hkv, D, sw_cfg.n_sink, w,
+                            seed=sw_cfg.seed + w, device=dev)
+        sw_ctx = [torch.from_numpy(wl.draft_ctx_for_step(sw_L, sw_k, j)).to(dev)
+                  for j in range(sw_k)]
+        sw_desc = spire.draft_desc(sdi.q, sdi.kv)
+        sw_ws = torch.empty(spire.spire_draft_workspace_bytes(sw_desc, sw_cfg.n_sink, w),
+                            dtype=torch.uint8, device=dev)
+        sw_out = torch.empty(sdi.q.shape, dtype=torch.float32, device=dev)
+
+        def call_sweep(j):
+            st = spire.spire_draft_sparse_attention(sdi.q, sdi.kv, sw_ctx[j], sw_cfg.n_sink, w,
+                                                    sw_desc, sw_out, sw_ws, sw_ws.numel(), sptr)
+            if st:
+                raise spire.SpireError(st, "spire_draft_sparse_attention")
+
+        for _ in range(max(3, args.warmup)):
+            for j in range(sw_k):
+                call_sweep(j)
+        torch.cuda.synchronize(dev)
+        if spire.spire_get_device_error(sw_ws, stream):
+            raise RuntimeError("device error word set by the draft sweep")
+        sw_ev = []
+        for s in range(max(1, min(args.steps, 50))):
+            for j in range(sw_k):
+                flush.fill_((s + j) & 0xff)     # each step streams its cache from HBM
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                call_sweep(j)
+                b.record(stream)
+                sw_ev.append((a, b))
+        torch.cuda.synchronize(dev)
+        round_ms = reduce_max([statistics.mean(a.elapsed_time(b) for a, b in sw_ev) * sw_k],
+                              dist, dev)[0]
+        sw_bytes = sum(draft_bytes(wl.draft_ctx_for_step(sw_L, sw_k, j), sw_S, Hq, Hkv, D)
+                       for j in range(sw_k))
+        sweep.append({"window": w, "n_sink": sw_cfg.n_sink, "cache_gb": sdi.kv.numel() * 2 / 1e9,
+                      "ms_per_round": round_ms,
+                      "draft_tokens_per_s": world * sw_B * sw_k / (round_ms * 1e-3),
+                      "gbs": sw_bytes / (round_ms * 1e-3) / 1e9,
+                      "frac": sw_bytes / (round_ms * 1e-3) / 1e9 / hbm_peak})
+        del sdi, sw_ctx, sw_ws, sw_out
+        torch.cuda.empty_cache()
+
     if rank != 0:
         if dist is not None:
             dist.barrier()
@@ -696,6 +748,11 @@ def spire_arm(args, cfg):
                        "gbs": tb / (tok_ms * 1e-3) / 1e9,
                        "frac": tb / (tok_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "mean_accepted": float(n_acc_h.mean()), "launches": 2},
+                   "draft_sweep": {
+                       "what": "B=%d, t log-uniform [4096, 262144], %d draft steps per round on "
+                               "one bounded cache per window, each step's cache streamed from "
+                               "HBM (L2 flushed before it)" % (sw_B, sw_k),
+                       "windows": sweep},
                    "draft_step_pipeline": {
                        "what": "one CUDA graph per round: %d steps x (%d layer attention calls + "
                                "one feedback append)" % (k, n_dl),
