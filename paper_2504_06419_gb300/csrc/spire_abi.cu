@@ -201,19 +201,24 @@ __global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n)
 // ------------------------------------------------------------- MagicDec gather
 // MagicDec's draft attends, with positions inside the reduced cache, to the
 // sink + window entries of the target's own paged cache (Section 3.1
-// footnote).  This kernel builds that reduced cache, one warp per item:
+// footnote).  This kernel builds that reduced cache, one warp per item; a
+// row of D bf16 sits in D/8 lanes, 16 bytes each, 32/(D/8) rows per step:
 //   sequence items  n_vis[b] = number of visible entries (0 if t is out of
 //                   range or a visible page id is outside the cache)
-//   row items       1/32 of the slots of (b, g): entry c at text position
-//                   p, K turned by (c - p) and rounded to bf16, V copied.  A
-//                   sink keeps its position (c = p) and every window entry
-//                   moves by the same s - w0, so a warp computes its lanes'
-//                   sine and cosine once and applies them to all its rows
-//   query items     q turned by the query's cache index n_vis - 1
+//   row items       1/8 of the visible entries of (b, g): entry c at text
+//                   position p, K turned by (c - p) and rounded to bf16, V
+//                   copied; the pages of a batch of rows are looked up first,
+//                   then all their K and V loads issue together.  A sink keeps
+//                   its position (c = p) and every window entry moves by the
+//                   same s - w0, so a lane computes the sines and cosines of
+//                   its eight elements once per item; the partner (d + D/2)
+//                   of an element comes from the lane D/16 away (shuffle)
+//   query items     q rows turned by their cache index n_vis - 1
 // Angles: reduced modulo 2 pi exactly in 64-bit fixed point (rope_sincos),
 // sine and cosine of the reduced angle in fp32 (positions up to 2^31 keep
-// their accuracy).
-constexpr int kMdParts = 32;          // row items per (sequence, KV head): few rows each
+// their accuracy).  The kernel also zeroes the attention's pair counters,
+// and the attention kernel follows it as its programmatic dependent.
+constexpr int kMdParts = 8;           // row items per (sequence, KV head)
 
 struct MdParams {
     const __nv_bfloat16* q;        // [B, Hq, D], not rotated
@@ -224,6 +229,7 @@ struct MdParams {
     __nv_bfloat16* kv;             // [B, 2, Hkv, S, D] reduced cache
     __nv_bfloat16* q_eff;          // [B, Hq, D]
     int32_t* n_vis;                // [B]
+    int32_t* cnt;                  // the attention's pair counters, zeroed here
     int B, Hq, Hkv, D, S, n_sink, window, max_pages, num_pages, rotate;
     uint64_t fturn[64];            // theta^(-2d/D) / (2 pi) as 64-bit fractions
 };
@@ -249,29 +255,54 @@ __device__ __forceinline__ void md_sincos(const uint64_t* turn, long long delta,
     rope_sincos(delta, turn[d], sn, cs);
 }
 
-// turn the pairs (d, d + D/2) of a row, lane handling d = lane + 32 i, by the
-// angles given as sines / cosines per i (identity: sn = 0, cs = 1), bf16 out
-__device__ __forceinline__ void md_turn_row(const __nv_bfloat16* src, __nv_bfloat16* dst,
-                                            const float* sn, const float* cs, int half,
-                                            int lane) {
+// A row of D bf16 is spread over D/8 lanes, eight consecutive elements (16
+// bytes) per lane; the pair partner (d + D/2) of a first-half lane's elements
+// sits in the lane D/16 further on.  Turns this lane's vector v given its
+// partner's w by the per-element sines / cosines:
+//   first half   v cs - w sn
+//   second half  v cs + w sn
+// rounding each result to bf16.
+__device__ __forceinline__ uint4 md_turn_vec(uint4 v, uint4 w, const float* sn, const float* cs,
+                                             bool first_half) {
+    const uint32_t a[4] = {v.x, v.y, v.z, v.w}, b[4] = {w.x, w.y, w.z, w.w};
+    uint32_t o[4];
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const int d = lane + 32 * i;
-        if (d >= half) break;
-        const float a0 = __bfloat162float(src[d]), a1 = __bfloat162float(src[d + half]);
-        dst[d] = __float2bfloat16_rn(a0 * cs[i] - a1 * sn[i]);
-        dst[d + half] = __float2bfloat16_rn(a1 * cs[i] + a0 * sn[i]);
+    for (int e = 0; e < 4; ++e) {
+        const float a0 = bf16lo_to_f32(a[e]), a1 = bf16hi_to_f32(a[e]);
+        const float b0 = bf16lo_to_f32(b[e]), b1 = bf16hi_to_f32(b[e]);
+        const float r0 = first_half ? a0 * cs[2 * e] - b0 * sn[2 * e] : a0 * cs[2 * e] + b0 * sn[2 * e];
+        const float r1 = first_half ? a1 * cs[2 * e + 1] - b1 * sn[2 * e + 1]
+                                    : a1 * cs[2 * e + 1] + b1 * sn[2 * e + 1];
+        o[e] = pack_bf16(r0, r1);
     }
+    return make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-__global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) {
+// sines / cosines of delta * freq for this lane's eight elements d0 .. d0 + 7
+__device__ __forceinline__ void md_lane_turn(const uint64_t* turn, long long delta, int d0,
+                                             float* sn, float* cs) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) md_sincos(turn, delta, d0 + e, &sn[e], &cs[e]);
+}
+
+constexpr int kMdBatch = 5;    // row steps whose loads a lane issues together
+
+__global__ void __launch_bounds__(256, 2) magicdec_gather_kernel(const MdParams p) {
     __shared__ uint64_t turn[64];
+    grid_dep_launch_dependents();      // the attention kernel waits for all of this grid
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < p.B * p.Hkv; i += gridDim.x * blockDim.x)
+        p.cnt[i] = 0;
     if (threadIdx.x < 64) turn[threadIdx.x] = p.fturn[threadIdx.x];
     __syncthreads();
-    const int lane = threadIdx.x & 31, half = p.D / 2;
+    const int lane = threadIdx.x & 31;
+    // lanes per row, rows per warp step, and this lane's place
+    const int LPR = p.D / 8, RPW = 32 / LPR, HL = LPR / 2;
+    const int jl = lane % LPR, sub = lane / LPR;
+    const bool first_half = jl < HL;
+    const int d0 = 8 * (jl % HL);
     const long long n_rows = (long long)p.B * p.Hkv * kMdParts;
-    const long long total = p.B + n_rows + (long long)p.B * p.Hq;
-    const int rpp = (p.S + kMdParts - 1) / kMdParts;         // slots per row item
+    const long long n_q = ((long long)p.B * p.Hq + RPW - 1) / RPW;
+    const long long total = p.B + n_rows + n_q;
     for (long long item = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5; item < total;
          item += ((long long)gridDim.x * blockDim.x) >> 5) {
         if (item < p.B) {
@@ -293,46 +324,80 @@ __global__ void __launch_bounds__(256) magicdec_gather_kernel(const MdParams p) 
             ok = __all_sync(0xffffffffu, ok);
             if (lane == 0) p.n_vis[b] = ok ? v.n : 0;
         } else if (item < p.B + n_rows) {
+            // row item: 1/kMdParts of the visible entries of one (sequence, KV head)
             long long r = item - p.B;
             const int part = (int)(r % kMdParts); r /= kMdParts;
             const int g = (int)(r % p.Hkv);
             const int b = (int)(r / p.Hkv);
             const MdVisible v = md_visible(p, p.ctx_lens[b]);
+            const int rpp = (v.n + kMdParts - 1) / kMdParts;
             const int c0 = part * rpp, c1 = min(v.n, c0 + rpp);
             if (c0 >= c1) continue;
-            // the window's common turn s - w0, once per lane
-            float wsn[2] = {0.f, 0.f}, wcs[2] = {1.f, 1.f};
-            const float zsn[2] = {0.f, 0.f}, ocs[2] = {1.f, 1.f};
-            if (p.rotate && v.s != v.w0)
+            // every window entry moves by the same s - w0: one table per lane
+            float wsn[8], wcs[8];
 #pragma unroll
-                for (int i = 0; i < 2; ++i)
-                    if (lane + 32 * i < half) md_sincos(turn, (long long)v.s - v.w0, lane + 32 * i, &wsn[i], &wcs[i]);
-#pragma unroll 2
-            for (int c = c0; c < c1; ++c) {
-                const bool sink = c < v.s;
-                const int pos = sink ? c : v.w0 + (c - v.s);
-                const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
-                if (id < 0 || id >= p.num_pages) continue;   // the sequence item reports it
-                const long long src = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * p.D;
-                const long long dk = ((((long long)b * 2 + 0) * p.Hkv + g) * p.S + c) * p.D;
-                const long long dv = ((((long long)b * 2 + 1) * p.Hkv + g) * p.S + c) * p.D;
-                md_turn_row(p.k_cache + src, p.kv + dk, sink ? zsn : wsn, sink ? ocs : wcs, half,
-                            lane);
-                for (int d = 2 * lane; d < p.D; d += 64)
-                    *reinterpret_cast<__nv_bfloat162*>(p.kv + dv + d) =
-                        *reinterpret_cast<const __nv_bfloat162*>(p.v_cache + src + d);
+            for (int e = 0; e < 8; ++e) { wsn[e] = 0.f; wcs[e] = 1.f; }
+            if (p.rotate && v.s != v.w0) md_lane_turn(turn, (long long)v.s - v.w0, d0, wsn, wcs);
+            for (int cb = c0; cb < c1; cb += RPW * kMdBatch) {
+                long long src[kMdBatch];
+                int row[kMdBatch];
+#pragma unroll
+                for (int i = 0; i < kMdBatch; ++i) {      // the entries' pages
+                    const int c = cb + i * RPW + sub;
+                    row[i] = -1;
+                    src[i] = 0;
+                    if (c < c1) {
+                        const int pos = c < v.s ? c : v.w0 + (c - v.s);
+                        const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
+                        if (id >= 0 && id < p.num_pages) {   // else the sequence item reports it
+                            row[i] = c;
+                            src[i] = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * p.D +
+                                     8 * jl;
+                        }
+                    }
+                }
+                uint4 kvk[kMdBatch], kvv[kMdBatch];
+#pragma unroll
+                for (int i = 0; i < kMdBatch; ++i) {      // all rows in flight together
+                    if (row[i] >= 0) {
+                        kvk[i] = *reinterpret_cast<const uint4*>(p.k_cache + src[i]);
+                        kvv[i] = *reinterpret_cast<const uint4*>(p.v_cache + src[i]);
+                    } else {
+                        kvk[i] = kvv[i] = make_uint4(0, 0, 0, 0);
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < kMdBatch; ++i) {
+                    const uint4 w = shfl_xor_u4(kvk[i], HL);
+                    if (row[i] < 0) continue;
+                    const bool sink = row[i] < v.s;
+                    const uint4 kt = (sink || !p.rotate) ? kvk[i]
+                                                          : md_turn_vec(kvk[i], w, wsn, wcs, first_half);
+                    const long long dk =
+                        ((((long long)b * 2 + 0) * p.Hkv + g) * p.S + row[i]) * p.D + 8 * jl;
+                    const long long dv =
+                        ((((long long)b * 2 + 1) * p.Hkv + g) * p.S + row[i]) * p.D + 8 * jl;
+                    *reinterpret_cast<uint4*>(p.kv + dk) = kt;
+                    *reinterpret_cast<uint4*>(p.kv + dv) = kvv[i];
+                }
             }
         } else {
-            const long long r = item - p.B - n_rows;
-            const int b = (int)(r / p.Hq);
+            // query item: RPW rows of q, each turned by its sequence's last cache index
+            const long long r = (item - p.B - n_rows) * RPW + sub;
+            const bool have = r < (long long)p.B * p.Hq;
+            const int b = have ? (int)(r / p.Hq) : 0;
             const MdVisible v = md_visible(p, p.ctx_lens[b]);
-            if (v.n == 0) continue;
-            float sn[2] = {0.f, 0.f}, cs[2] = {1.f, 1.f};
-            if (p.rotate && v.n > 1)
-#pragma unroll
-                for (int i = 0; i < 2; ++i)
-                    if (lane + 32 * i < half) md_sincos(turn, v.n - 1, lane + 32 * i, &sn[i], &cs[i]);
-            md_turn_row(p.q + r * p.D, p.q_eff + r * p.D, sn, cs, half, lane);
+            uint4 x = make_uint4(0, 0, 0, 0);
+            if (have) x = *reinterpret_cast<const uint4*>(p.q + r * p.D + 8 * jl);
+            const uint4 w = shfl_xor_u4(x, HL);
+            if (!have || v.n == 0) continue;
+            uint4 y = x;
+            if (p.rotate && v.n > 1) {
+                float sn[8], cs[8];
+                md_lane_turn(turn, v.n - 1, d0, sn, cs);
+                y = md_turn_vec(x, w, sn, cs, first_half);
+            }
+            *reinterpret_cast<uint4*>(p.q_eff + r * p.D + 8 * jl) = y;
         }
     }
 }
@@ -352,11 +417,14 @@ MdLayout md_layout(const spire_attn_desc* d, int S) {
     return l;
 }
 
-// Shared launch sequence for both calls.
+// Launches the attention for one call: a one-CTA kernel zeroing the pair
+// counters, then the attention kernel as its programmatic dependent.  With
+// counters_zeroed the kernel launched just before (which must have zeroed
+// them, and may have written ctx_lens) is the attention kernel's dependency.
 spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorMap& tv,
                  const int32_t* block_table, const int32_t* ctx_lens, int kp1,
                  const spire_attn_desc* d, int cap, float* out, void* workspace,
-                 cudaStream_t stream) {
+                 cudaStream_t stream, bool counters_zeroed = false) {
     DeviceInfo di;
     spire_status st = device_info(&di);
     if (st != SPIRE_OK) return st;
@@ -386,13 +454,16 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     ap.num_pages = mode == kModeVerify ? d->num_pages : 0;
     ap.cap = cap;
     ap.mode = mode;
+    ap.wait_first = counters_zeroed ? 1 : 0;
     ap.sl2 = static_cast<float>(static_cast<double>(d->softmax_scale) * kLog2e);
 
     CUtensorMap tq;
     if (!encode_q_map(&tq, q, D, d->num_q_heads, uint64_t(B) * kp1, ap.G, kp1))
         return SPIRE_ERR_CUDA;
-    zero_counters_kernel<<<1, 256, 0, stream>>>(ap.cnt, B * Hkv);
-    if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+    if (!counters_zeroed) {
+        zero_counters_kernel<<<1, 256, 0, stream>>>(ap.cnt, B * Hkv);
+        if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+    }
     const int ctas = di.sms < kMaxCtas ? di.sms : kMaxCtas;
     const int mt = (R + 15) / 16;
     // tcgen05 path when a KV head serves enough query rows to make QK^T and PV
@@ -540,6 +611,10 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
     mp.kv = reinterpret_cast<__nv_bfloat16*>(ws + l.kv);
     mp.q_eff = reinterpret_cast<__nv_bfloat16*>(ws + l.q);
     mp.n_vis = reinterpret_cast<int32_t*>(ws + l.nvis);
+    // the attention's workspace starts the MagicDec workspace: its pair
+    // counters are zeroed by the gather, so no separate zeroing launch
+    mp.cnt = reinterpret_cast<int32_t*>(
+        ws + ws_layout(desc->batch, desc->num_kv_heads, rows_per_kv_head(desc, 1), desc->head_dim).cnt);
     mp.B = desc->batch;
     mp.Hq = desc->num_q_heads;
     mp.Hkv = desc->num_kv_heads;
@@ -556,16 +631,19 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
         mp.fturn[d] = mp.rotate
                           ? rope_turn_fixed(std::pow((double)rope_theta, -2.0 * d / desc->head_dim))
                           : 0;
-    const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * kMdParts + mp.Hq);
+    const int rpw = 32 / (desc->head_dim / 8);     // query rows per warp item
+    const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * kMdParts) +
+                            ((long long)mp.B * mp.Hq + rpw - 1) / rpw;
     long long blocks = (items * 32 + 255) / 256;
     if (blocks > 32LL * di.sms) blocks = 32LL * di.sms;
-    magicdec_gather_kernel<<<(unsigned)blocks, 256, 0, s>>>(mp);
+    magicdec_gather_kernel<<<(unsigned)blocks, 256, 0, s>>>(mp);   // a plain launch: after all prior work
     if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
 
     CUtensorMap tkv;
     const uint64_t planes = uint64_t(desc->batch) * 2u * uint64_t(desc->num_kv_heads);
     if (!encode_kv_map(&tkv, mp.kv, desc->head_dim, uint64_t(S), planes)) return SPIRE_ERR_CUDA;
-    return run(kModeDraft, mp.q_eff, tkv, tkv, nullptr, mp.n_vis, 1, desc, S, out, workspace, s);
+    return run(kModeDraft, mp.q_eff, tkv, tkv, nullptr, mp.n_vis, 1, desc, S, out, workspace, s,
+               true);
 }
 
 int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {

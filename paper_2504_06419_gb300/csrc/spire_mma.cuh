@@ -103,6 +103,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     for (int i = threadIdx.x; i < 2 * C::QBUF / 16; i += blockDim.x)
         reinterpret_cast<uint4*>(sbase + C::OFF_Q)[i] = make_uint4(0u, 0u, 0u, 0u);
     fence_proxy_async();
+    if (p.wait_first) grid_dep_wait();   // ctx_lens are that kernel's output
     sched_setup(p, sh);   // ends with __syncthreads()
     // the arrival counters were zeroed by the kernel launched just before
     grid_dep_wait();

@@ -213,6 +213,15 @@ __device__ __forceinline__ void st_dsmem_f32(uint32_t a, float v) {
     asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
 }
 
+// A 16-byte vector from lane (lane ^ mask) of the warp (all lanes take part).
+__device__ __forceinline__ uint4 shfl_xor_u4(uint4 v, int mask) {
+    v.x = __shfl_xor_sync(0xffffffffu, v.x, mask);
+    v.y = __shfl_xor_sync(0xffffffffu, v.y, mask);
+    v.z = __shfl_xor_sync(0xffffffffu, v.z, mask);
+    v.w = __shfl_xor_sync(0xffffffffu, v.w, mask);
+    return v;
+}
+
 // Named barrier over `count` threads (a multiple of 32).
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");

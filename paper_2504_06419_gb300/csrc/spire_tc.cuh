@@ -132,6 +132,7 @@ __global__ void __launch_bounds__(224, 1)
         tmem_relinquish();
         tc_fence_before();
     }
+    if (p.wait_first) grid_dep_wait();   // ctx_lens are that kernel's output
     sched_setup(p, sh);   // ends with __syncthreads()
     tc_fence_after();
     // the arrival counters were zeroed by the kernel launched just before
