@@ -179,8 +179,10 @@ def test_append_rejects_bad_args(spire):
 
 def test_tokens_workspace_and_host_checks(spire):
     E = spire._lib
-    assert spire.spire_verify_tokens_workspace_bytes(64, 4, 128256) == 512 + 64 * 16 * 24
-    assert spire.spire_verify_tokens_workspace_bytes(1, 0, 1) == 512 + 24
+    # header and error word, one 8-byte accept record per sequence (256-byte
+    # aligned), one 24-byte partial per 4096-entry chunk
+    assert spire.spire_verify_tokens_workspace_bytes(64, 4, 128256) == 512 + 512 + 64 * 32 * 24
+    assert spire.spire_verify_tokens_workspace_bytes(1, 0, 1) == 512 + 256 + 24
     for bad in [(0, 4, 100), (1, -1, 100), (1, 32, 100), (1, 4, 0), (70000, 1, 10)]:
         assert spire.spire_verify_tokens_workspace_bytes(*bad) == 0
     good = 1 << 20
