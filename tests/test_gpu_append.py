@@ -109,6 +109,10 @@ CASES = [
     ("two_token_blocks", list(range(300)), 3, 1, 256, 2, 128, 16, 48, 0.0),
     ("no_sink_ring", [5, 6, 7, 8, 70000, 1 << 30], 1, 1, 128, 1, 128, 0, 8, 10000.0),
     ("draft_2x4096", list(range(7000, 7064)), 3, 2, 4096, 8, 128, 16, 512, 10000.0),
+    # 16 activations: 16 tokens per block, one MMA of N = 256
+    ("sixteen_activations", list(range(3, 60, 3)), 16, 2, 128, 2, 64, 2, 30, 10000.0),
+    # 5 K splits (clusters of 5) over 48-token blocks: 9 or 10 tokens per rank
+    ("five_splits_uneven", list(range(0, 504, 7)), 5, 1, 320, 3, 64, 4, 20, 500000.0),
 ]
 
 

@@ -34,8 +34,10 @@ CASES = [
     # batch, k, vocab
     (1, 0, 7),            # plain sampling, scalar loads
     (3, 1, 1001),         # scalar loads (V % 4 != 0), one chunk
-    (64, 4, 32000),       # 16-byte loads, four chunks
-    (17, 8, 8193),        # a chunk of one entry
+    (64, 4, 32000),       # bulk copies: 8 units of 4096 per sequence, a 3328-entry tail
+    (17, 8, 8193),        # scalar loads, a chunk of one entry
+    (2, 0, 4096),         # plain sampling on the bulk-copy path: one unit, no q row
+    (5, 3, 100),          # one unit of 100 entries (a 400-byte copy)
     (64, 4, 128256),      # a Llama 3 sized vocabulary
 ]
 
