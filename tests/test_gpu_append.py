@@ -113,6 +113,10 @@ CASES = [
     ("sixteen_activations", list(range(3, 60, 3)), 16, 2, 128, 2, 64, 2, 30, 10000.0),
     # 5 K splits (clusters of 5) over 48-token blocks: 9 or 10 tokens per rank
     ("five_splits_uneven", list(range(0, 504, 7)), 5, 1, 320, 3, 64, 4, 20, 500000.0),
+    # 20 row tiles: clusters of 7 asked for, fewer if the GPU cannot hold 20 of them
+    ("twenty_tiles", [11, 12, 13, 14, 15, 16, 17, 18], 3, 1, 512, 10, 128, 8, 8, 10000.0),
+    # one token, one K block: a single CTA without a split
+    ("one_token_one_block", [4], 2, 1, 64, 1, 128, 2, 6, 10000.0),
 ]
 
 
