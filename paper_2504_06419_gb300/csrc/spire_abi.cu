@@ -230,7 +230,12 @@ struct MdParams {
     __nv_bfloat16* q_eff;          // [B, Hq, D]
     int32_t* n_vis;                // [B]
     int32_t* cnt;                  // the attention's pair counters, zeroed here
+    float* out;                    // fused path: [B, Hq, D]
+    int32_t* header;               // fused path: error words (one per merge CTA)
+    int32_t* err;
     int B, Hq, Hkv, D, S, n_sink, window, max_pages, num_pages, rotate;
+    int G;                         // query heads per KV head
+    float sl2;                     // softmax_scale * log2(e)
     uint64_t fturn[64];            // theta^(-2d/D) / (2 pi) as 64-bit fractions
 };
 
@@ -402,9 +407,222 @@ __global__ void __launch_bounds__(256, 2) magicdec_gather_kernel(const MdParams 
     }
 }
 
+// ------------------------------------------------------------- MagicDec, fused
+// For up to 8 query heads per KV head the draft attention is computed where
+// the rows are read, in fp32 on the CUDA cores (4 FLOP per K/V byte: no
+// contraction worth the tensor cores).  One CTA per (sequence, KV head) pair
+// (a grid-stride loop over pairs): warp w of 4 takes 1/4 of the pair's visible
+// entries as the gather does (a batch of page lookups, then all the batch's
+// 16-byte K and V loads), turns and rounds the keys, and keeps for each of the
+// G query rows (turned by n - 1 and rounded, held by every row group of the
+// warp) a running maximum, sum and output in base 2; the warp's row groups
+// merge by shuffles, the four warps through shared memory in warp order, and
+// the CTA writes the G output rows.  A bad page, or a context length out of
+// range, gives NaN rows and SPIRE_DEVERR_CTX_LEN, as on the gather path.
+constexpr int kMfWarps = 4;        // one wave: 512 pairs fit as 4 CTAs per SM
+constexpr int kMfBatch = 3;      // row steps whose loads a lane issues together
+
+template <int D, int GP>
+__global__ void __launch_bounds__(32 * kMfWarps, GP <= 4 ? 4 : 2)
+    magicdec_fused_kernel(const MdParams p) {
+    __shared__ uint64_t turn[64];
+    __shared__ float sm_o[kMfWarps][GP][D];
+    __shared__ float sm_ml[kMfWarps][GP][2];
+    __shared__ int sm_bad;
+    __shared__ uint32_t cta_err;
+    if (threadIdx.x < 64) turn[threadIdx.x] = p.fturn[threadIdx.x];
+    if (threadIdx.x == 0) cta_err = 0;
+    __syncthreads();
+    constexpr int LPR = D / 8, RPW = 32 / LPR, HL = LPR / 2;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int jl = lane % LPR, sub = lane / LPR;
+    const bool first_half = jl < HL;
+    const int d0 = 8 * (jl % HL);
+    const long long pairs = (long long)p.B * p.Hkv;
+    for (long long bg = blockIdx.x; bg < pairs; bg += gridDim.x) {
+        const int g = (int)(bg % p.Hkv), b = (int)(bg / p.Hkv);
+        const MdVisible v = md_visible(p, p.ctx_lens[b]);
+        const int rpp = (v.n + kMfWarps - 1) / kMfWarps;
+        const int c0 = warp * rpp, c1 = min(v.n, c0 + rpp);
+        if (threadIdx.x == 0) sm_bad = v.n == 0;
+        // the query rows of this KV head, turned by n - 1 and rounded to bf16
+        float qv[GP][8];
+        {
+            float sn[8], cs[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) { sn[e] = 0.f; cs[e] = 1.f; }
+            const bool turnq = p.rotate && v.n > 1;
+            if (turnq) md_lane_turn(turn, v.n - 1, d0, sn, cs);
+#pragma unroll
+            for (int h = 0; h < GP; ++h) {
+                uint4 x = make_uint4(0, 0, 0, 0);
+                if (h < p.G)
+                    x = *reinterpret_cast<const uint4*>(
+                        p.q + ((long long)b * p.Hq + (long long)g * p.G + h) * D + 8 * jl);
+                const uint4 w = shfl_xor_u4(x, HL);
+                const uint4 y = turnq ? md_turn_vec(x, w, sn, cs, first_half) : x;
+                const uint32_t a[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    qv[h][2 * e] = bf16lo_to_f32(a[e]);
+                    qv[h][2 * e + 1] = bf16hi_to_f32(a[e]);
+                }
+            }
+        }
+        float wsn[8], wcs[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { wsn[e] = 0.f; wcs[e] = 1.f; }
+        if (p.rotate && v.s != v.w0) md_lane_turn(turn, (long long)v.s - v.w0, d0, wsn, wcs);
+        float m[GP], l[GP], o[GP][8];
+#pragma unroll
+        for (int h = 0; h < GP; ++h) {
+            m[h] = -INFINITY;
+            l[h] = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
+        }
+        bool bad = false;
+        for (int cb = c0; cb < c1; cb += RPW * kMfBatch) {
+            long long src[kMfBatch];
+            int row[kMfBatch];
+#pragma unroll
+            for (int i = 0; i < kMfBatch; ++i) {      // the entries' pages
+                const int c = cb + i * RPW + sub;
+                row[i] = -1;
+                src[i] = 0;
+                if (c < c1) {
+                    const int pos = c < v.s ? c : v.w0 + (c - v.s);
+                    const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
+                    if (id >= 0 && id < p.num_pages) {
+                        row[i] = c;
+                        src[i] = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * D + 8 * jl;
+                    } else {
+                        bad = true;
+                    }
+                }
+            }
+            uint4 kvk[kMfBatch], kvv[kMfBatch];
+#pragma unroll
+            for (int i = 0; i < kMfBatch; ++i) {      // all rows in flight together
+                if (row[i] >= 0) {
+                    kvk[i] = *reinterpret_cast<const uint4*>(p.k_cache + src[i]);
+                    kvv[i] = *reinterpret_cast<const uint4*>(p.v_cache + src[i]);
+                } else {
+                    kvk[i] = kvv[i] = make_uint4(0, 0, 0, 0);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < kMfBatch; ++i) {
+                const uint4 w = shfl_xor_u4(kvk[i], HL);
+                const bool valid = row[i] >= 0;
+                const bool sink = row[i] < v.s;
+                const uint4 kt = (sink || !p.rotate) ? kvk[i]
+                                                      : md_turn_vec(kvk[i], w, wsn, wcs, first_half);
+                const uint32_t ka[4] = {kt.x, kt.y, kt.z, kt.w};
+                const uint32_t va[4] = {kvv[i].x, kvv[i].y, kvv[i].z, kvv[i].w};
+                float kf[8], vf[8];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    kf[2 * e] = bf16lo_to_f32(ka[e]);
+                    kf[2 * e + 1] = bf16hi_to_f32(ka[e]);
+                    vf[2 * e] = bf16lo_to_f32(va[e]);
+                    vf[2 * e + 1] = bf16hi_to_f32(va[e]);
+                }
+#pragma unroll
+                for (int h = 0; h < GP; ++h) {
+                    float sc = 0.f;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) sc = fmaf(qv[h][e], kf[e], sc);
+#pragma unroll
+                    for (int off = HL; off >= 1; off >>= 1)   // the row's LPR lanes
+                        sc += __shfl_xor_sync(0xffffffffu, sc, off);
+                    if (!valid) continue;
+                    const float s2 = sc * p.sl2;
+                    const float mn = fmaxf(m[h], s2);
+                    const float corr = exp2f(m[h] - mn), pe = exp2f(s2 - mn);
+                    m[h] = mn;
+                    l[h] = fmaf(l[h], corr, pe);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) o[h][e] = fmaf(o[h][e], corr, pe * vf[e]);
+                }
+            }
+        }
+        // the warp's row groups hold different entries: merge them
+#pragma unroll
+        for (int off = LPR; off < 32; off <<= 1) {
+#pragma unroll
+            for (int h = 0; h < GP; ++h) {
+                const float m2 = __shfl_xor_sync(0xffffffffu, m[h], off);
+                const float l2 = __shfl_xor_sync(0xffffffffu, l[h], off);
+                const float mn = fmaxf(m[h], m2);
+                const float c1s = mn == -INFINITY ? 0.f : exp2f(m[h] - mn);
+                const float c2s = mn == -INFINITY ? 0.f : exp2f(m2 - mn);
+                l[h] = l[h] * c1s + l2 * c2s;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float o2 = __shfl_xor_sync(0xffffffffu, o[h][e], off);
+                    o[h][e] = o[h][e] * c1s + o2 * c2s;
+                }
+                m[h] = mn;
+            }
+        }
+        if (__any_sync(0xffffffffu, bad) && lane == 0) sm_bad = 1;
+        if (sub == 0) {
+#pragma unroll
+            for (int h = 0; h < GP; ++h) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) sm_o[warp][h][8 * jl + e] = o[h][e];
+                if (jl == 0) {
+                    sm_ml[warp][h][0] = m[h];
+                    sm_ml[warp][h][1] = l[h];
+                }
+            }
+        }
+        __syncthreads();
+        // the warps' results, in warp order, for the G rows
+        const bool pbad = sm_bad != 0;
+        if (pbad && threadIdx.x == 0) cta_err |= kErrCtxLen;
+        for (int i = threadIdx.x; i < p.G * D; i += blockDim.x) {
+            const int h = i / D, d = i % D;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kMfWarps; ++w) M = fmaxf(M, sm_ml[w][h][0]);
+            float L = 0.f, O = 0.f;
+#pragma unroll
+            for (int w = 0; w < kMfWarps; ++w) {
+                const float mw = sm_ml[w][h][0];
+                if (mw == -INFINITY) continue;
+                const float sc = exp2f(mw - M);
+                L = fmaf(sm_ml[w][h][1], sc, L);
+                O = fmaf(sm_o[w][h][d], sc, O);
+            }
+            p.out[((long long)b * p.Hq + (long long)g * p.G + h) * D + d] =
+                (pbad || !(L > 0.f)) ? NAN : O / L;
+        }
+        __syncthreads();                         // shared memory is reused by the next pair
+    }
+    // one error word per CTA: every CTA writes its own, nothing needs clearing
+    if (threadIdx.x == 0) {
+        p.err[blockIdx.x] = (int32_t)cta_err;
+        if (blockIdx.x == 0) p.header[0] = (int32_t)gridDim.x;
+    }
+}
+
 struct MdLayout {
     size_t draft, kv, q, nvis, total;
 };
+
+// query heads per KV head padded to 1, 2, 4 or 8 (fused path), 0 if above 8
+int md_fused_gp(const spire_attn_desc* d) {
+    const int G = d->num_q_heads / d->num_kv_heads;
+    return G <= 1 ? 1 : G <= 2 ? 2 : G <= 4 ? 4 : G <= 8 ? 8 : 0;
+}
+
+// fused path workspace: header word | error words (one per CTA)
+size_t md_fused_bytes(const spire_attn_desc* d) {
+    if (md_fused_gp(d) == 0) return 0;
+    return kHeaderBytes + align256(size_t(kMaxCtas) * 4);
+}
 
 MdLayout md_layout(const spire_attn_desc* d, int S) {
     MdLayout l{};
@@ -566,7 +784,8 @@ size_t spire_magicdec_workspace_bytes(const spire_attn_desc* desc, int32_t n_sin
     if (check_common(desc) != SPIRE_OK || n_sink < 0 || window < 1 ||
         (long long)n_sink + window > 65536)
         return 0;
-    return md_layout(desc, n_sink + window).total;
+    const size_t gather = md_layout(desc, n_sink + window).total, fused = md_fused_bytes(desc);
+    return gather > fused ? gather : fused;
 }
 
 spire_status spire_magicdec_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -595,7 +814,8 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
         return SPIRE_ERR_INVALID_ARG;
     const int S = n_sink + window;
     const MdLayout l = md_layout(desc, S);
-    if (!workspace || !aligned(workspace, 256) || ws_bytes < l.total) return SPIRE_ERR_WORKSPACE;
+    const size_t need = l.total > md_fused_bytes(desc) ? l.total : md_fused_bytes(desc);
+    if (!workspace || !aligned(workspace, 256) || ws_bytes < need) return SPIRE_ERR_WORKSPACE;
     DeviceInfo di;
     st = device_info(&di);
     if (st != SPIRE_OK) return st;
@@ -631,6 +851,26 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
         mp.fturn[d] = mp.rotate
                           ? rope_turn_fixed(std::pow((double)rope_theta, -2.0 * d / desc->head_dim))
                           : 0;
+    const int gp = md_fused_gp(desc);
+    if (gp != 0) {
+        // up to 8 query heads per KV head: the fused kernel and its merge
+        mp.G = desc->num_q_heads / desc->num_kv_heads;
+        mp.sl2 = static_cast<float>(static_cast<double>(desc->softmax_scale) * kLog2e);
+        mp.header = reinterpret_cast<int32_t*>(ws);
+        mp.err = reinterpret_cast<int32_t*>(ws + kHeaderBytes);
+        mp.out = out;
+        const long long pairs = (long long)mp.B * mp.Hkv;
+        const long long fblocks = pairs < kMaxCtas ? pairs : kMaxCtas;   // one error word each
+        void (*fk)(MdParams) = nullptr;
+#define SPIRE_MD_CASE(DD, GG) \
+    if (desc->head_dim == DD && gp == GG) fk = magicdec_fused_kernel<DD, GG>;
+        SPIRE_MD_CASE(64, 1) SPIRE_MD_CASE(64, 2) SPIRE_MD_CASE(64, 4) SPIRE_MD_CASE(64, 8)
+        SPIRE_MD_CASE(128, 1) SPIRE_MD_CASE(128, 2) SPIRE_MD_CASE(128, 4) SPIRE_MD_CASE(128, 8)
+#undef SPIRE_MD_CASE
+        if (!fk) return SPIRE_ERR_UNSUPPORTED;
+        fk<<<(unsigned)fblocks, 32 * kMfWarps, 0, s>>>(mp);   // after all prior work
+        return cudaGetLastError() == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
+    }
     const int rpw = 32 / (desc->head_dim / 8);     // query rows per warp item
     const long long items = (long long)mp.B * (1 + (long long)mp.Hkv * kMdParts) +
                             ((long long)mp.B * mp.Hq + rpw - 1) / rpw;
