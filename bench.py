@@ -738,7 +738,8 @@ def spire_arm(args, cfg):
                    "magicdec_draft_step": {
                        "what": "spire_magicdec_attention: sink %d + window %d over the target's "
                                "paged cache, keys and query re-turned to cache positions "
-                               "(gather + draft attention launches)" % (md_sink, md_win),
+                               "(one fused launch for up to 8 query heads per KV head)"
+                               % (md_sink, md_win),
                        "us": md_ms * 1e3, "algorithmic_bytes": md_bytes,
                        "gbs": md_bytes / (md_ms * 1e-3) / 1e9,
                        "spire_draft_step_us": d_ms / k * 1e3},
