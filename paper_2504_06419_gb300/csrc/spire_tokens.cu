@@ -16,17 +16,16 @@
 //   tokens_accept_kernel    one warp per sequence: j from the k gathered
 //                           probabilities (a ballot), and the bad-token flag;
 //                           clears the device error word.
-//   tokens_stream_kernel    its programmatic dependent, one or two CTAs per
-//                           SM walking (sequence, chunk of 4096 entries)
-//                           units: a producer warp copies the chunk's rows
-//                           p_{j+1}, q_{j+1} (only if j < k) and E into a
-//                           four-stage shared-memory ring with bulk async
-//                           copies (the copy engine keeps ~200 KB per SM in
-//                           flight, where 16-byte loads stall on the L1's
-//                           outstanding-miss limit near 25 GB/s per SM), and
-//                           eight consumer warps reduce the best (score,
-//                           index) key of the residual and of p alone; one
-//                           partial per unit.
+//   tokens_stream_kernel    its programmatic dependent, four CTAs per SM
+//                           walking (sequence, chunk of 4096 entries) units:
+//                           a producer warp copies the chunk's rows p_{j+1},
+//                           q_{j+1} (only if j < k) and E into a four-stage
+//                           shared-memory ring (1024 entries per stage) with
+//                           bulk async copies, and eight consumer warps
+//                           reduce the best (score, index) key of the
+//                           residual and of p alone, dividing exactly only
+//                           where an estimate reaches the warp's best so far;
+//                           one partial per unit.
 //   tokens_finalize_kernel  one warp per sequence: the best key over the
 //                           chunks (the maximum is unique, so the order of the
 //                           reduction cannot matter), the emitted tokens and j.
@@ -51,8 +50,9 @@ namespace {
 constexpr int kTokThreads = 256;
 constexpr int kTokChunk = 8192;          // vocabulary entries per CTA (race kernel)
 constexpr int kTokUnit = 4096;           // vocabulary entries per unit (stream kernel)
-constexpr int kTokSub = 2048;            // entries per stage and row (8 KB)
+constexpr int kTokSub = 1024;            // entries per stage and row (4 KB), a multiple of 1024
 constexpr int kTokStages = 4;
+constexpr int kTokStreamCtas = 4;        // CTAs per SM (the register limit at 288 threads)
 constexpr int kTokConsumers = 8;         // consumer warps of the stream kernel
 constexpr int kTokStreamThreads = 32 * (kTokConsumers + 1);
 constexpr int kTokMaxK = 31;
@@ -96,6 +96,19 @@ __device__ __forceinline__ unsigned long long race_key(float w, float e, int v) 
 __device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
     return a > b ? a : b;
 }
+
+// Approximate reciprocal (the hardware's, relative error below 2^-22 for
+// normal inputs; a subnormal input gives infinity, which the filter passes).
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
+// An estimate w * rcp(E) is within a factor (1 +- 2^-21) of the exact w / E
+// (reciprocal 2^-22, product 2^-24): below best * (1 - 2^-20) it cannot reach
+// the best score.
+constexpr float kTokFilter = 1.0f - 0x1p-20f;
 
 __global__ void __launch_bounds__(kTokThreads) tokens_race_kernel(const TokParams p) {
     const int s = blockIdx.x, b = blockIdx.y;
@@ -238,7 +251,7 @@ __global__ void __launch_bounds__(128) tokens_accept_kernel(const TokParams p) {
     if (lane == 0) p.acc[b] = a;
 }
 
-__global__ void __launch_bounds__(kTokStreamThreads, 2) tokens_stream_kernel(const TokParams p) {
+__global__ void __launch_bounds__(kTokStreamThreads, kTokStreamCtas) tokens_stream_kernel(const TokParams p) {
     extern __shared__ __align__(128) uint8_t tsm[];   // [stage][p | q | E rows of kTokSub]
     __shared__ __align__(8) uint64_t bars[2 * kTokStages];
     __shared__ unsigned long long s_kr[kTokConsumers], s_kp[kTokConsumers];
@@ -305,6 +318,7 @@ __global__ void __launch_bounds__(kTokStreamThreads, 2) tokens_stream_kernel(con
         const bool res = j < k;
         const int c1 = min(V, (c + 1) * kTokUnit);
         unsigned long long kr = 0, kp = 0;
+        float thr_p = 0.f, thr_r = 0.f;             // filters on the estimates
         int flags = 0;
         for (int v0 = c * kTokUnit; v0 < c1; v0 += kTokSub) {
             const int n = min(kTokSub, c1 - v0);
@@ -316,8 +330,8 @@ __global__ void __launch_bounds__(kTokStreamThreads, 2) tokens_stream_kernel(con
             const float* sq = reinterpret_cast<const float*>(tsm + s * STAGE + ROW);
             const float* se = reinterpret_cast<const float*>(tsm + s * STAGE + 2 * ROW);
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int i = 4 * ct + h * (kTokSub / 2);
+            for (int h = 0; h < kTokSub / 1024; ++h) {   // 4 entries per consumer thread and pass
+                const int i = 4 * ct + h * 1024;
                 if (i >= n) continue;
                 const float4 pv = *reinterpret_cast<const float4*>(sp + i);
                 const float4 ev = *reinterpret_cast<const float4*>(se + i);
@@ -331,16 +345,36 @@ __global__ void __launch_bounds__(kTokStreamThreads, 2) tokens_stream_kernel(con
                         flags |= (int)kTokErrValue;
                         continue;
                     }
-                    if (pa[e] > 0.f) kp = umax64(kp, race_key(pa[e], ea[e], v));
+                    // w * rcp(E) is within 2^-21 of w / E, so an entry whose
+                    // estimate is below thr cannot reach (or tie) the best
+                    // score: only the rest pay the exact division
+                    const float rcp = rcp_approx(ea[e]);
+                    if (pa[e] > 0.f && pa[e] * rcp >= thr_p) {
+                        kp = umax64(kp, race_key(pa[e], ea[e], v));
+                        thr_p = fmaxf(thr_p, __uint_as_float((uint32_t)(kp >> 32)) * kTokFilter);
+                    }
                     if (res) {
                         const float w = __fsub_rn(pa[e], qa[e]);
-                        if (w > 0.f) kr = umax64(kr, race_key(w, ea[e], v));
+                        if (w > 0.f && w * rcp >= thr_r) {
+                            kr = umax64(kr, race_key(w, ea[e], v));
+                            thr_r = fmaxf(thr_r, __uint_as_float((uint32_t)(kr >> 32)) * kTokFilter);
+                        }
                     }
                 }
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_empty + 8 * s);
             if (++s == kTokStages) { s = 0; ph ^= 1; }
+            // the warp's best so far sets every lane's filter: an entry below
+            // it cannot be the maximum, and lanes that agree do not diverge
+            unsigned long long wp = kp, wr = kr;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                wp = umax64(wp, __shfl_xor_sync(0xffffffffu, wp, o));
+                wr = umax64(wr, __shfl_xor_sync(0xffffffffu, wr, o));
+            }
+            thr_p = __uint_as_float((uint32_t)(wp >> 32)) * kTokFilter;
+            thr_r = __uint_as_float((uint32_t)(wr >> 32)) * kTokFilter;
         }
         // the unit's best keys over the consumer threads
 #pragma unroll
@@ -499,7 +533,8 @@ spire_status spire_verify_tokens(const float* p, const float* q, const int32_t* 
     tokens_accept_kernel<<<(unsigned)((batch + 3) / 4), 128, 0, st>>>(tp);
     if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
     const long long units = (long long)batch * tp.S;
-    const long long grid = units < 2LL * sms ? units : 2LL * sms;   // two CTAs per SM
+    const long long ctas = (long long)kTokStreamCtas * sms;
+    const long long grid = units < ctas ? units : ctas;
     if (launch_dependent(tokens_stream_kernel, dim3((unsigned)grid), dim3(kTokStreamThreads),
                          (size_t)kStreamSmem, st, tp) != cudaSuccess)
         return SPIRE_ERR_CUDA;
