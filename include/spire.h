@@ -31,6 +31,15 @@
  * Conventions common to every call
  *   - All tensor arguments are DEVICE pointers, owned by the caller; the
  *     library keeps no pointer after a call returns and allocates nothing.
+ *     One exception: `out` of spire_verify_attention(_noalloc),
+ *     spire_draft_sparse_attention and spire_magicdec_attention may also be
+ *     pinned host memory mapped into the device's address space
+ *     (cudaHostAlloc / cudaHostRegister memory on a system with unified
+ *     addressing, where the host pointer is valid on the device).  Those
+ *     kernels only store to `out`, with plain stores, so the results reach
+ *     the host without a separate copy (zero-copy; over NVLink-C2C on a
+ *     Grace host) and are visible there once the stream has reached the end
+ *     of the call.
  *   - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
  *     NULL is the legacy default stream).  Only spire_get_device_error
  *     synchronises.

@@ -218,3 +218,47 @@ def test_draft_slot_matches_oracle(spire):
     for ns, w in [(0, 1), (4, 64), (16, 512), (32, 2048), (16, 4096)]:
         for p in list(range(0, 3000, 7)) + [10 ** 6 - 1, 262143]:
             assert spire.spire_draft_slot(p, ns, w) == oracle.draft_slot(p, ns, w)
+
+
+# ---------------------------------------------------------------- zero-copy outputs
+def _pinned_like(t):
+    return torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+
+
+@pytest.mark.parametrize("case", [([700, 5], 0, 8, 8, 128),        # warp-MMA kernel, R = 1
+                                  ([4100, 70, 1000], 4, 32, 8, 128),  # tcgen05, four query copies
+                                  ([9, 3000, 200], 8, 64, 8, 128)],   # tcgen05, one copy (72 rows)
+                         ids=["mma", "tc4", "tc1"])
+def test_verify_output_in_pinned_host_memory(spire, case):
+    """`out` may be mapped pinned host memory: the kernels store into it
+    directly and the result equals the one written to device memory."""
+    L, k, Hq, Hkv, D = case
+    vi = wl.make_verify(L, k, Hq, Hkv, D, seed=61, device=DEV)
+    ref = parity.gpu_verify(spire, vi)
+    host = _pinned_like(ref)
+    host.fill_(float("nan"))
+    spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, k,
+                           softmax_scale=vi.scale, out=host)
+    torch.cuda.synchronize()
+    assert torch.equal(host, ref.cpu())
+
+
+def test_draft_and_magicdec_output_in_pinned_host_memory(spire):
+    di = wl.make_draft([3, 600, 20000], 32, 8, 128, 16, 512, seed=62, device=DEV)
+    ref = spire.draft_attention(di.q, di.kv, di.ctx_lens, 16, 512)
+    host = _pinned_like(ref)
+    host.fill_(float("nan"))
+    spire.draft_attention(di.q, di.kv, di.ctx_lens, 16, 512, out=host)
+    torch.cuda.synchronize()
+    assert torch.equal(host, ref.cpu())
+    for Hq, Hkv in ((32, 8), (64, 1)):          # fused kernel (G <= 8), gather + attention
+        vi = wl.make_verify([5, 900, 9000], 0, Hq, Hkv, 128, seed=63, device=DEV)
+        q = vi.q[:, 0].contiguous()
+        ref = spire.magicdec_attention(q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens,
+                                       4, 256, 10000.0)
+        host = _pinned_like(ref)
+        host.fill_(float("nan"))
+        spire.magicdec_attention(q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, 4, 256,
+                                 10000.0, out=host)
+        torch.cuda.synchronize()
+        assert torch.equal(host, ref.cpu()), (Hq, Hkv)
