@@ -186,6 +186,17 @@ def reduce_max(values, dist=None, device=None):
     return [float(x) for x in t.cpu().tolist()]
 
 
+def cta_balance(times):
+    """Per-SM busy time of one attention call from its per-CTA timing record."""
+    busy = [(e - b) / 1e3 for b, e in times]
+    mean = statistics.mean(busy)
+    first = min(b for b, _ in times)
+    return {"ctas": len(times), "busy_us_mean": mean, "busy_us_max": max(busy),
+            "busy_us_min": min(busy), "max_over_mean": max(busy) / mean if mean > 0 else None,
+            "start_spread_us": (max(b for b, _ in times) - first) / 1e3,
+            "span_us": (max(e for _, e in times) - first) / 1e3}
+
+
 def job_value(tokens_per_rank, world, step_ms):
     """Whole-job throughput: every rank processes its own batch (weak scaling)."""
     return world * tokens_per_rank / (step_ms * 1e-3)
@@ -238,10 +249,14 @@ def run_oracle_sample(cfg, n_seq, threads):
 
 
 def oracle_sample_size(cfg, target_s=15.0, threads=None):
-    """Sequences of the workload that keep the oracle leg near target_s."""
+    """Sequences of the workload that keep the oracle leg near target_s: the
+    oracle's time grows with the context it reads, so the first sequence's
+    time per context token is scaled by the cumulative lengths."""
+    L = wl.sample_ctx_lens(cfg).astype(np.float64)
     dt, _ = run_oracle_sample(cfg, 1, threads)
-    n = int(max(1, min(cfg.batch, math.floor(target_s / max(dt, 1e-3)))))
-    return n
+    per_token = max(dt, 1e-3) / L[0]
+    n = int(np.searchsorted(np.cumsum(L) * per_token, target_s, side="right"))
+    return int(max(1, min(cfg.batch, n)))
 
 
 def reference_arm(args, cfg):
@@ -492,6 +507,14 @@ def spire_arm(args, cfg):
         e2e_ms.append(a.elapsed_time(b))
     e2e_val = job_value(tokens, world, reduce_max([statistics.mean(e2e_ms)], dist, dev)[0])
 
+    # ---- load balance: per-SM busy time of one verify and one draft call
+    flush.fill_(1)
+    call_verify()
+    bal_v = cta_balance(spire.spire_get_cta_times(ws_v, ws_v.numel()))
+    flush.fill_(2)
+    call_draft(0)
+    bal_d = cta_balance(spire.spire_get_cta_times(ws_d, ws_d.numel()))
+
     # ---- draft-step pipeline: a draft with n_dl = 2 layers (3 activations mixed,
     # d_model = Hq * D); each step attends on every layer's cache, then appends
     # the new feedback-memory entry to every cache (spire_feedback_append)
@@ -691,6 +714,11 @@ def spire_arm(args, cfg):
         cpu = {"value": tok / dt, "unit": "tokens/s", "cores": threads, "kind": "oracle",
                "sample": "first %d of %d sequences, verify + %d draft steps, fp64 C oracle, "
                          "%.1f s" % (n_seq, cfg.batch, k, dt)}
+        # the same oracle on one core, on a smaller sample
+        n1 = oracle_sample_size(cfg, target_s=5.0, threads=1)
+        dt1, tok1 = run_oracle_sample(cfg, n1, 1)
+        cpu["single_core"] = {"value": tok1 / dt1, "unit": "tokens/s", "cores": 1,
+                              "sample": "first %d sequences, %.1f s" % (n1, dt1)}
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -729,6 +757,11 @@ def spire_arm(args, cfg):
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "launches": 1},
                    "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
+                   "load_balance": {
+                       "what": "per-CTA %globaltimer record (spire_get_cta_times) of one verify "
+                               "call and one draft call after an L2 flush: busy = first tile "
+                               "to last merge, one CTA per SM",
+                       "verify": bal_v, "draft_step": bal_d},
                    "magicdec_draft_step": {
                        "what": "spire_magicdec_attention: sink %d + window %d over the target's "
                                "paged cache, keys and query re-turned to cache positions "
@@ -742,7 +775,7 @@ def spire_arm(args, cfg):
                        "us": tok_ms * 1e3, "algorithmic_bytes": tb,
                        "gbs": tb / (tok_ms * 1e-3) / 1e9,
                        "frac": tb / (tok_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
-                       "mean_accepted": float(n_acc_h.mean()), "launches": 2},
+                       "mean_accepted": float(n_acc_h.mean()), "launches": 3},
                    "draft_sweep": {
                        "what": "B=%d, t log-uniform [4096, 262144], %d draft steps per round on "
                                "one bounded cache per window, each step's cache streamed from "

@@ -41,8 +41,8 @@
  *     Grace host) and are visible there once the stream has reached the end
  *     of the call.
  *   - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
- *     NULL is the legacy default stream).  Only spire_get_device_error
- *     synchronises.
+ *     NULL is the legacy default stream).  Only spire_get_device_error and
+ *     spire_get_cta_times synchronise.
  *   - Arguments that can be checked on the host are checked before anything is
  *     launched; a failing check returns a status and launches nothing.
  *   - Values that live on the device (ctx_lens, block_table) are checked by
@@ -167,7 +167,8 @@ SPIRE_API spire_status spire_verify_attention(const void *q, const void *k_cache
  *   - All calls share the one array: calls that may overlap on the GPU (on
  *     different streams, or from different threads) race and must not be
  *     issued.  The array keeps the last call's contents; each call clears what
- *     must start at zero.  spire_get_device_error is not available for it.
+ *     must start at zero.  spire_get_device_error and spire_get_cta_times are
+ *     not available for it.
  */
 SPIRE_API spire_status spire_verify_attention_noalloc(const void *q, const void *k_cache,
                                                       const void *v_cache,
@@ -386,6 +387,24 @@ SPIRE_API int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
  */
 SPIRE_API spire_status spire_get_device_error(const void *workspace, int32_t *code_out,
                                     void *stream);
+
+/*
+ * spire_get_cta_times -- the per-CTA timing record of the most recent
+ * spire_verify_attention or spire_draft_sparse_attention call that used
+ * `workspace` (ws_bytes of it): for each of the call's n CTAs (one per SM, in
+ * CTA order) two %globaltimer readings in nanoseconds, when the CTA started
+ * its first tile (after the launch dependency) and when it finished its last
+ * output or merge.  The difference is that SM's busy time; the split of the
+ * KV range gives every CTA the same number of tiles (within one), so the
+ * spread shows how evenly the time follows.  Synchronises `stream`, writes n
+ * to *n_out and the first min(n, max_ctas) pairs to ns_out[2i], ns_out[2i+1]
+ * (host memory).  Returns SPIRE_ERR_WORKSPACE if ws_bytes cannot hold the
+ * record of n CTAs.  The record is meaningless after any other call on the
+ * same workspace (which does not write it).
+ */
+SPIRE_API spire_status spire_get_cta_times(const void *workspace, size_t ws_bytes,
+                                 uint64_t *ns_out, int32_t max_ctas, int32_t *n_out,
+                                 void *stream);
 
 /* spire_status_string -- static, human-readable name of a status. */
 SPIRE_API const char *spire_status_string(spire_status status);

@@ -43,6 +43,7 @@ EXPORTED = (
     "spire_verify_tokens",
     "spire_draft_slot",
     "spire_get_device_error",
+    "spire_get_cta_times",
     "spire_status_string",
 )
 
@@ -115,6 +116,9 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_draft_slot.argtypes = [I64, I32, I32]
     lib.spire_get_device_error.restype = ctypes.c_int
     lib.spire_get_device_error.argtypes = [P, ctypes.POINTER(I32), P]
+    lib.spire_get_cta_times.restype = ctypes.c_int
+    lib.spire_get_cta_times.argtypes = [P, SZ, ctypes.POINTER(ctypes.c_uint64), I32,
+                                        ctypes.POINTER(I32), P]
     lib.spire_status_string.restype = ctypes.c_char_p
     lib.spire_status_string.argtypes = [ctypes.c_int]
     return lib
@@ -236,6 +240,18 @@ def spire_get_device_error(workspace, stream=None) -> int:
     if st != SPIRE_OK:
         raise SpireError(st, "spire_get_device_error")
     return int(code.value)
+
+
+def spire_get_cta_times(workspace, ws_bytes, max_ctas=1024, stream=None):
+    """Per-CTA (start_ns, end_ns) of the last verify / draft call on `workspace`."""
+    buf = (ctypes.c_uint64 * (2 * max_ctas))()
+    n = ctypes.c_int32(0)
+    st = LIB.spire_get_cta_times(_ptr(workspace), int(ws_bytes), buf, int(max_ctas),
+                                 ctypes.byref(n), _stream(stream, workspace))
+    if st != SPIRE_OK:
+        raise SpireError(st, "spire_get_cta_times")
+    m = min(n.value, max_ctas)
+    return [(int(buf[2 * i]), int(buf[2 * i + 1])) for i in range(m)]
 
 
 def status_string(status: int) -> str:

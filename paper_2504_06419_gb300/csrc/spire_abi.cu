@@ -24,17 +24,23 @@ constexpr double kLog2e = 1.4426950408889634;  // log2(e): softmax runs in base 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct WsLayout {
-    size_t err, cnt, part_lse, part_o, total;
+    size_t err, stamps, cnt, part_lse, part_o, total;
 };
 
-// header (grid size of the last call) | per-CTA error words | per-pair
-// arrival counters | partial slots (two per CTA: a CTA range cuts at most
-// its first and its last pair).
+// Offset of the per-CTA timing record: fixed, so that spire_get_cta_times
+// needs only the workspace pointer.
+constexpr size_t kStampsOffset = kHeaderBytes + ((size_t(kMaxCtas) * 4 + 255) & ~size_t(255));
+static_assert(kStampsOffset % 256 == 0, "the timing record starts a 256-byte block");
+
+// header (grid size of the last call) | per-CTA error words | per-CTA timing
+// record | per-pair arrival counters | partial slots (two per CTA: a CTA
+// range cuts at most its first and its last pair).
 WsLayout ws_layout(long long B, long long Hkv, long long R, long long D) {
     const long long slots = 2LL * kMaxCtas;
     WsLayout w{};
     size_t off = kHeaderBytes;
     w.err = off;      off += align256(size_t(kMaxCtas) * 4);
+    w.stamps = off;   off += align256(size_t(kMaxCtas) * 16);
     w.cnt = off;      off += align256(size_t(B * Hkv) * 4);
     w.part_lse = off; off += align256(size_t(slots * R) * 4);
     w.part_o = off;   off += align256(size_t(slots * R * D) * 4);
@@ -660,6 +666,7 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     ap.header = reinterpret_cast<int32_t*>(ws);
     ap.err = reinterpret_cast<int32_t*>(ws + w.err);
     ap.cnt = reinterpret_cast<int32_t*>(ws + w.cnt);
+    ap.stamps = reinterpret_cast<unsigned long long*>(ws + w.stamps);
     ap.part_lse = reinterpret_cast<float*>(ws + w.part_lse);
     ap.part_o = reinterpret_cast<float*>(ws + w.part_o);
     ap.B = B;
@@ -910,6 +917,27 @@ spire_status spire_get_device_error(const void* workspace, int32_t* code_out, vo
     int32_t v = 0;
     for (int c = 0; c < n; ++c) v |= buf[c];
     *code_out = v;
+    return SPIRE_OK;
+}
+
+spire_status spire_get_cta_times(const void* workspace, size_t ws_bytes, uint64_t* ns_out,
+                                 int32_t max_ctas, int32_t* n_out, void* stream) {
+    if (!workspace || !n_out || max_ctas < 0 || (max_ctas > 0 && !ns_out))
+        return SPIRE_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t n = 0;
+    if (ws_bytes < kHeaderBytes) return SPIRE_ERR_WORKSPACE;
+    if (cudaMemcpyAsync(&n, workspace, sizeof(n), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return SPIRE_ERR_CUDA;
+    if (n < 0 || n > kMaxCtas) n = 0;
+    if (kStampsOffset + (size_t)n * 16 > ws_bytes) return SPIRE_ERR_WORKSPACE;
+    const int m = n < max_ctas ? n : max_ctas;
+    if (m > 0 && (cudaMemcpyAsync(ns_out, static_cast<const char*>(workspace) + kStampsOffset,
+                                  (size_t)m * 16, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+                  cudaStreamSynchronize(s) != cudaSuccess))
+        return SPIRE_ERR_CUDA;
+    *n_out = n;
     return SPIRE_OK;
 }
 

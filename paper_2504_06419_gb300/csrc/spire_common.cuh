@@ -70,6 +70,8 @@ struct AttnParams {
     int32_t* header;           // [0]: grid size of the last call
     int32_t* err;              // [kMaxCtas]: error bits of each CTA of the last call
     int32_t* cnt;              // [B * Hkv]: segment arrival counters, zero at launch
+    unsigned long long* stamps;  // [2 * kMaxCtas]: per CTA, %globaltimer when its first tile
+                                 // starts and when its last merge is done (last call)
     float* part_o;             // [2 * kMaxCtas * R, D]
     float* part_lse;           // [2 * kMaxCtas * R]
     int32_t B, Hq, Hkv, G, kp1, R;

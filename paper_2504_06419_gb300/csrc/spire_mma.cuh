@@ -107,6 +107,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     sched_setup(p, sh);   // ends with __syncthreads()
     // the arrival counters were zeroed by the kernel launched just before
     grid_dep_wait();
+    if (threadIdx.x == 0) p.stamps[2 * blockIdx.x] = globaltimer_ns();
 
     if (warp == C::NW) {
         // ------------------------------------------------------ producer
@@ -129,7 +130,10 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
                 return;
             }
             const int4 i0 = scr_info[2 * sb], i1 = scr_info[2 * sb + 1];
-            if (i1.y) return;                          // the consumers have finished
+            if (i1.y) {                                // the consumers have finished
+                if (lane == 0) p.stamps[2 * blockIdx.x + 1] = globaltimer_ns();
+                return;
+            }
             const int cb = i0.x, cg = i0.y, cslot = i0.z, cnseg = i0.w, cfirst = i1.x;
             const float* so = scr_o + sb * C::SCR_BUF;
             const float2* sml = scr_ml + sb * C::NW * C::SR;

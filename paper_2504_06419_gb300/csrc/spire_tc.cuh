@@ -137,6 +137,7 @@ __global__ void __launch_bounds__(224, 1)
     tc_fence_after();
     // the arrival counters were zeroed by the kernel launched just before
     grid_dep_wait();
+    if (threadIdx.x == 0) p.stamps[2 * blockIdx.x] = globaltimer_ns();
     const uint32_t tmem = misc[0];
     uint32_t err = 0;
 
@@ -525,6 +526,7 @@ __global__ void __launch_bounds__(224, 1)
     }
     if (err) atomicOr(&p.err[blockIdx.x], (int)err);
     __syncthreads();
+    if (threadIdx.x == 0) p.stamps[2 * blockIdx.x + 1] = globaltimer_ns();
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem, C::TMEM_COLS);

@@ -31,7 +31,7 @@ def test_header_declares_the_boundary():
         "spire_feedback_append_workspace_bytes", "spire_feedback_append",
         "spire_verify_tokens_workspace_bytes", "spire_verify_tokens",
         "spire_magicdec_workspace_bytes", "spire_magicdec_attention",
-        "spire_get_device_error", "spire_status_string"]), names
+        "spire_get_device_error", "spire_get_cta_times", "spire_status_string"]), names
 
 
 def test_library_exports_every_declared_symbol(spire):
@@ -223,3 +223,16 @@ def test_magicdec_host_checks(spire):
     assert call(q=good + 8) == E.SPIRE_ERR_INVALID_ARG
     assert call(desc=_desc(spire, page_size=32)) == E.SPIRE_ERR_UNSUPPORTED
     assert call(window=70000) == E.SPIRE_ERR_UNSUPPORTED
+
+
+def test_cta_times_host_checks(spire):
+    """Argument errors of spire_get_cta_times come back before any CUDA call."""
+    lib = spire._lib.LIB
+    n = ctypes.c_int32(-1)
+    buf = (ctypes.c_uint64 * 4)()
+    assert lib.spire_get_cta_times(None, 1 << 20, buf, 2, ctypes.byref(n), None) == 1
+    assert lib.spire_get_cta_times(256, 1 << 20, buf, 2, None, None) == 1
+    assert lib.spire_get_cta_times(256, 1 << 20, None, 2, ctypes.byref(n), None) == 1
+    assert lib.spire_get_cta_times(256, 1 << 20, buf, -1, ctypes.byref(n), None) == 1
+    assert lib.spire_get_cta_times(256, 255, buf, 2, ctypes.byref(n), None) == 3
+    assert n.value == -1

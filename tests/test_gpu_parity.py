@@ -262,3 +262,31 @@ def test_draft_and_magicdec_output_in_pinned_host_memory(spire):
                                  10000.0, out=host)
         torch.cuda.synchronize()
         assert torch.equal(host, ref.cpu()), (Hq, Hkv)
+
+
+# ---------------------------------------------------------------- per-CTA timing record
+def test_cta_times_cover_every_cta(spire):
+    L = [4100, 70, 1000, 2049, 30000, 5]
+    for k, Hq, Hkv in ((4, 32, 8), (0, 8, 8)):        # tcgen05 and warp-MMA kernels
+        vi = wl.make_verify(L, k, Hq, Hkv, 128, seed=64, device=DEV)
+        desc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+        nb = spire.spire_verify_workspace_bytes(desc, k)
+        ws = torch.full((nb,), 0xff, dtype=torch.uint8, device=DEV)
+        spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, k,
+                               workspace=ws)
+        t = spire.spire_get_cta_times(ws, nb)
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        assert len(t) == min(sms, 512)
+        starts = np.array([a for a, _ in t], dtype=np.float64)
+        ends = np.array([b for _, b in t], dtype=np.float64)
+        assert np.all(ends >= starts)
+        assert ends.max() - starts.min() < 1e9             # one call: well under a second
+        with pytest.raises(spire.SpireError):
+            spire.spire_get_cta_times(ws, 1024)           # too small for the record
+    di = wl.make_draft([3, 600, 20000], 32, 8, 128, 16, 512, seed=65, device=DEV)
+    desc = spire.draft_desc(di.q, di.kv)
+    nb = spire.spire_draft_workspace_bytes(desc, 16, 512)
+    ws = torch.full((nb,), 0xff, dtype=torch.uint8, device=DEV)
+    spire.draft_attention(di.q, di.kv, di.ctx_lens, 16, 512, workspace=ws)
+    t = spire.spire_get_cta_times(ws, nb)
+    assert len(t) >= 1 and all(b >= a for a, b in t)
