@@ -290,3 +290,32 @@ def test_cta_times_cover_every_cta(spire):
     spire.draft_attention(di.q, di.kv, di.ctx_lens, 16, 512, workspace=ws)
     t = spire.spire_get_cta_times(ws, nb)
     assert len(t) >= 1 and all(b >= a for a, b in t)
+
+
+# ---------------------------------------------------------------- workspace reuse
+def test_workspace_needs_no_initialisation_and_survives_reuse(spire):
+    """Every call resets the merge counters it uses before its attention
+    kernel reads them, so any starting content works and one workspace can
+    serve calls of other shapes in turn (ordered on one stream)."""
+    L = [30000, 4100, 70]                       # three sequences: every pair is split
+    vi = wl.make_verify(L, 4, 32, 8, 128, seed=66, device=DEV)
+    di = wl.make_draft([5, 9000, 600, 40, 3000], 32, 8, 128, 16, 512, seed=67, device=DEV)
+    ref_v = parity.gpu_verify(spire, vi)
+    ref_d = parity.gpu_draft(spire, di)
+    vdesc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+    ddesc = spire.draft_desc(di.q, di.kv)
+    nb = max(spire.spire_verify_workspace_bytes(vdesc, 4),
+             spire.spire_draft_workspace_bytes(ddesc, 16, 512))
+    g = torch.Generator(device="cpu").manual_seed(68)
+    fills = [torch.zeros(nb, dtype=torch.uint8), torch.full((nb,), 255, dtype=torch.uint8),
+             torch.randint(0, 256, (nb,), dtype=torch.uint8, generator=g)]
+    for fill in fills:
+        ws = fill.to(DEV)
+        for _ in range(2):
+            out = spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table,
+                                         vi.ctx_lens, 4, workspace=ws)
+            dout = spire.draft_attention(di.q, di.kv, di.ctx_lens, 16, 512, workspace=ws)
+            torch.cuda.synchronize()
+            assert torch.equal(out, ref_v)
+            assert torch.equal(dout, ref_d)
+            assert spire.spire_get_device_error(ws) == 0
