@@ -197,10 +197,14 @@ bool encode_3d_bf16_map(CUtensorMap* map, const void* base, uint64_t inner, uint
 
 namespace {
 
-// Zeroes the per-pair arrival counters; lets the attention kernel launched
-// after it start its prologue at once (programmatic dependent launch).
+// Zeroes the per-pair arrival counters.  A programmatic dependent of the
+// kernel before it (one CTA, it fits beside a running attention CTA): it lets
+// the attention kernel after it launch at once and zeroes the counters only
+// when the kernel before has completed, so back-to-back calls hide both
+// launches behind the previous call's tail.
 __global__ void __launch_bounds__(256) zero_counters_kernel(int32_t* cnt, int n) {
     grid_dep_launch_dependents();
+    grid_dep_wait();
     for (int i = threadIdx.x; i < n; i += blockDim.x) cnt[i] = 0;
 }
 
@@ -642,9 +646,11 @@ MdLayout md_layout(const spire_attn_desc* d, int S) {
 }
 
 // Launches the attention for one call: a one-CTA kernel zeroing the pair
-// counters, then the attention kernel as its programmatic dependent.  With
-// counters_zeroed the kernel launched just before (which must have zeroed
-// them, and may have written ctx_lens) is the attention kernel's dependency.
+// counters, then the attention kernel, each a programmatic dependent of the
+// kernel before it (each waits for that kernel to complete before it touches
+// global memory).  With counters_zeroed the kernel launched just before
+// (which must have zeroed them, and may have written ctx_lens) is the
+// attention kernel's dependency.
 spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorMap& tv,
                  const int32_t* block_table, const int32_t* ctx_lens, int kp1,
                  const spire_attn_desc* d, int cap, float* out, void* workspace,
@@ -679,15 +685,15 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     ap.num_pages = mode == kModeVerify ? d->num_pages : 0;
     ap.cap = cap;
     ap.mode = mode;
-    ap.wait_first = counters_zeroed ? 1 : 0;
     ap.sl2 = static_cast<float>(static_cast<double>(d->softmax_scale) * kLog2e);
 
     CUtensorMap tq;
     if (!encode_q_map(&tq, q, D, d->num_q_heads, uint64_t(B) * kp1, ap.G, kp1))
         return SPIRE_ERR_CUDA;
     if (!counters_zeroed) {
-        zero_counters_kernel<<<1, 256, 0, stream>>>(ap.cnt, B * Hkv);
-        if (cudaGetLastError() != cudaSuccess) return SPIRE_ERR_CUDA;
+        if (launch_dependent(zero_counters_kernel, dim3(1), dim3(256), 0, stream, ap.cnt,
+                             B * Hkv) != cudaSuccess)
+            return SPIRE_ERR_CUDA;
     }
     const int ctas = di.sms < kMaxCtas ? di.sms : kMaxCtas;
     const int mt = (R + 15) / 16;

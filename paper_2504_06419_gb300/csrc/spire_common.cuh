@@ -78,7 +78,6 @@ struct AttnParams {
     int32_t max_pages, num_pages;  // verify
     int32_t cap;                   // draft: cache slots S = n_sink + window
     int32_t mode;
-    int32_t wait_first;            // ctx_lens come from the kernel launched just before
     float sl2;                     // softmax_scale * log2(e)
 };
 

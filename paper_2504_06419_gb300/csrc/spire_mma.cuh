@@ -96,17 +96,21 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
             mbar_init(bar_sempty + 8 * b, 1);
         }
         fence_barrier_init();
-        if (blockIdx.x == 0) p.header[0] = gridDim.x;
-        p.err[blockIdx.x] = 0;
     }
     // Q rows past R are never loaded: keep them zero for the whole kernel
     for (int i = threadIdx.x; i < 2 * C::QBUF / 16; i += blockDim.x)
         reinterpret_cast<uint4*>(sbase + C::OFF_Q)[i] = make_uint4(0u, 0u, 0u, 0u);
     fence_proxy_async();
-    if (p.wait_first) grid_dep_wait();   // ctx_lens are that kernel's output
-    sched_setup(p, sh);   // ends with __syncthreads()
-    // the arrival counters were zeroed by the kernel launched just before
+    // Global memory is touched only after the kernel before (the counter reset,
+    // which itself waits for all earlier work) has completed; then the next
+    // call's kernels may launch and start their prologue on freed SMs.
     grid_dep_wait();
+    grid_dep_launch_dependents();
+    if (threadIdx.x == 0) {
+        if (blockIdx.x == 0) p.header[0] = gridDim.x;
+        p.err[blockIdx.x] = 0;
+    }
+    sched_setup(p, sh);   // ends with __syncthreads()
     if (threadIdx.x == 0) p.stamps[2 * blockIdx.x] = globaltimer_ns();
 
     if (warp == C::NW) {

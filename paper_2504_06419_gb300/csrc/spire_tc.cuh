@@ -120,8 +120,6 @@ __global__ void __launch_bounds__(224, 1)
         mbar_init(bar_drain, 1);
         mbar_init(bar_drain + 8, 1);
         fence_barrier_init();
-        if (blockIdx.x == 0) p.header[0] = gridDim.x;
-        p.err[blockIdx.x] = 0;
     }
     // Q rows of padding stay zero for the whole kernel
     for (int i = threadIdx.x; i < C::QBUF / 16; i += blockDim.x)
@@ -132,11 +130,17 @@ __global__ void __launch_bounds__(224, 1)
         tmem_relinquish();
         tc_fence_before();
     }
-    if (p.wait_first) grid_dep_wait();   // ctx_lens are that kernel's output
+    // Global memory is touched only after the kernel before (the counter reset,
+    // which itself waits for all earlier work) has completed; then the next
+    // call's kernels may launch and start their prologue on freed SMs.
+    grid_dep_wait();
+    grid_dep_launch_dependents();
+    if (threadIdx.x == 0) {
+        if (blockIdx.x == 0) p.header[0] = gridDim.x;
+        p.err[blockIdx.x] = 0;
+    }
     sched_setup(p, sh);   // ends with __syncthreads()
     tc_fence_after();
-    // the arrival counters were zeroed by the kernel launched just before
-    grid_dep_wait();
     if (threadIdx.x == 0) p.stamps[2 * blockIdx.x] = globaltimer_ns();
     const uint32_t tmem = misc[0];
     uint32_t err = 0;

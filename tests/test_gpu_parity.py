@@ -319,3 +319,41 @@ def test_workspace_needs_no_initialisation_and_survives_reuse(spire):
             assert torch.equal(out, ref_v)
             assert torch.equal(dout, ref_d)
             assert spire.spire_get_device_error(ws) == 0
+
+
+# ---------------------------------------------------------------- split invariance
+def test_split_plan_invariance(spire):
+    """The same sequences under different split plans (alone, with a few
+    companions, inside a large batch: every call cuts the KV range across
+    the SMs differently) agree to fp32 rounding with one another and with the
+    oracle.  The caches are shared; only q, the block-table rows and ctx_lens
+    of the chosen sequences change."""
+    L = [20000, 5000] + [3000] * 40
+    vi = wl.make_verify(L, 4, 32, 8, 128, seed=69, device=DEV)
+    full = parity.gpu_verify(spire, vi)
+
+    def sub(idx):
+        idx_t = torch.as_tensor(idx, dtype=torch.long, device=DEV)
+        v = wl.VerifyInputs(q=vi.q[idx_t].contiguous(), k_cache=vi.k_cache, v_cache=vi.v_cache,
+                            block_table=vi.block_table[idx_t].contiguous(),
+                            ctx_lens=vi.ctx_lens[idx_t].contiguous(), k=vi.k)
+        return parity.gpu_verify(spire, v)
+
+    alone = sub([0])
+    pair = sub([1, 0])
+    ref, _ = parity.oracle_verify(wl.VerifyInputs(
+        q=vi.q[:2], k_cache=vi.k_cache, v_cache=vi.v_cache, block_table=vi.block_table[:2],
+        ctx_lens=vi.ctx_lens[:2], k=vi.k))
+    for got, row in ((full[0], 0), (alone[0], 0), (pair[1], 0), (full[1], 1), (pair[0], 1)):
+        parity.assert_close(got.cpu().numpy(), ref[row], "split plan, sequence %d" % row)
+    for a, b in ((full[0], alone[0]), (full[0], pair[1]), (full[1], pair[0])):
+        rel, mx = parity.errors(a.cpu().numpy(), b.cpu().numpy())
+        assert rel <= 1e-5 and mx <= 1e-5, (rel, mx)
+    # draft: one sequence alone and inside a batch of 64
+    di = wl.make_draft([9000] + [2000] * 63, 32, 8, 128, 16, 512, seed=70, device=DEV)
+    dfull = parity.gpu_draft(spire, di)
+    d1 = wl.DraftInputs(q=di.q[:1].contiguous(), kv=di.kv[:1].contiguous(),
+                        ctx_lens=di.ctx_lens[:1].contiguous(), n_sink=16, window=512)
+    done = parity.gpu_draft(spire, d1)
+    rel, mx = parity.errors(dfull[0].cpu().numpy(), done[0].cpu().numpy())
+    assert rel <= 1e-5 and mx <= 1e-5, (rel, mx)
