@@ -19,6 +19,8 @@ namespace spire {
 namespace {
 
 constexpr size_t kHeaderBytes = 256;
+constexpr int kHeadTc = 4;    // per-pair fixed cost of the tcgen05 attention kernel, in tiles
+constexpr int kHeadMma = 1;   // the same for the warp-MMA attention kernel
 constexpr double kLog2e = 1.4426950408889634;  // log2(e): softmax runs in base 2
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -701,6 +703,11 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     // real contractions; the warp-MMA path for the few-row draft step, whose
     // short pairs favour its lighter per-pair epilogue (measured on GB300)
     const bool use_tc = R > 8;
+    // the split's per-pair weight, from per-CTA timings on GB300 (busy time
+    // against planned tiles and segments): ~4 tiles for the tcgen05 kernel,
+    // whose softmax warps run the segment epilogue and the merge, ~1 for the
+    // warp-MMA kernel, whose epilogue warp works beside the stream
+    ap.head = use_tc ? kHeadTc : kHeadMma;
     cudaError_t e;
     const int nc = R <= 32 ? 4 : (R <= 64 ? 2 : 1);   // query copies of the tcgen05 kernel
     if (use_tc)

@@ -8,9 +8,9 @@
 // query rows per KV head against a run of 64-token K/V tiles.
 //
 // Decomposition.  The unit of work is one 64-token tile of one
-// (sequence b, KV head g) pair, plus kHead units of fixed cost per pair (its
+// (sequence b, KV head g) pair, plus `head` units of fixed cost per pair (its
 // query load and epilogue).  Pairs are laid end to end in the order (b, g),
-// each as [kHead head units | T tile units], numbered globally 0..W-1.  CTA c
+// each as [head units | T tile units], numbered globally 0..W-1.  CTA c
 // of a grid of N takes the contiguous range [floor(cW/N), floor((c+1)W/N)):
 // every SM gets the same work whatever the spread of lengths, counting the
 // per-pair cost that many short pairs add.  A pair whose
@@ -35,7 +35,9 @@ namespace spire {
 
 constexpr int kPage = 64;        // tokens per K/V tile (and per page)
 constexpr int kMaxCtas = 512;    // grid cap; the workspace holds 2 partial slots per CTA
-constexpr int kHead = 4;         // per-pair fixed cost, in tiles (tuned on GB300, ragged lengths)
+// Per-pair fixed cost in tile units (AttnParams::head), chosen per kernel by
+// the host: a pair's start and end (Q load, epilogue, output or partial) cost
+// the tcgen05 kernel about four tiles, the warp-MMA kernel about one.
 
 constexpr uint32_t kErrCtxLen = 1u;
 constexpr uint32_t kErrPageId = 2u;
@@ -79,6 +81,7 @@ struct AttnParams {
     int32_t cap;                   // draft: cache slots S = n_sink + window
     int32_t mode;
     float sl2;                     // softmax_scale * log2(e)
+    int32_t head;                  // per-pair fixed cost in tile units (the split's weights)
 };
 
 // Tiles of sequence b: ceil(visible length / 64); a sequence whose length
@@ -157,7 +160,7 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
     for (int b = threadIdx.x; b < p.B; b += blockDim.x) {
         int le;
         bool ok;
-        acc += seq_tiles(p, p.ctx_lens[b], &le, &ok) + kHead;
+        acc += seq_tiles(p, p.ctx_lens[b], &le, &ok) + p.head;
         bad |= !ok;
     }
     const long long units = block_sum(acc, sh);
@@ -176,7 +179,7 @@ __device__ inline void sched_setup(const AttnParams& p, SchedShared* sh) {
         const int b = base + threadIdx.x;
         int le;
         bool ok;
-        const long long U = b < p.B ? seq_tiles(p, p.ctx_lens[b], &le, &ok) + kHead : 0;
+        const long long U = b < p.B ? seq_tiles(p, p.ctx_lens[b], &le, &ok) + p.head : 0;
         long long chunk;
         const long long P = carry + block_excl_scan(U, sh, &chunk);
         if (b < p.B && lo < hi && P * p.Hkv <= lo && lo < (P + U) * p.Hkv) {
@@ -223,11 +226,11 @@ struct TileWalker {
         x = at; b = sb; g = 0; t = 0; first = true;
         T = seq_tiles(p, p.ctx_lens[b], &leff, &valid);
         const long long off = x - pb;
-        const int U = T + kHead;
+        const int U = T + p.head;
         g = (int)(off / U);
         const int u = (int)(off - (long long)g * U);
-        if (u < kHead) x += kHead - u;             // a part starting in a pair's head
-        else t = u - kHead;
+        if (u < p.head) x += p.head - u;             // a part starting in a pair's head
+        else t = u - p.head;
     }
 
     __device__ void init(const AttnParams& p, const SchedShared& sh, bool tail_first) {
@@ -241,11 +244,11 @@ struct TileWalker {
         int le1;
         bool ok1;
         const int T1 = seq_tiles(p, p.ctx_lens[sh.b1], &le1, &ok1);
-        const int U1 = T1 + kHead;
+        const int U1 = T1 + p.head;
         const long long g1 = (sh.hi - 1 - sh.p1) / U1;
         const long long pstart = sh.p1 + g1 * U1;
-        if (tail_first && pstart > sh.lo && sh.hi - 1 - pstart >= kHead && pstart + U1 > sh.hi) {
-            seek(p, pstart + kHead, sh.b1, sh.p1);  // the tail pair first
+        if (tail_first && pstart > sh.lo && sh.hi - 1 - pstart >= p.head && pstart + U1 > sh.hi) {
+            seek(p, pstart + p.head, sh.b1, sh.p1);  // the tail pair first
             rest_end = pstart;
         } else {
             seek(p, sh.lo, sh.b0, sh.p0);
@@ -260,7 +263,7 @@ struct TileWalker {
         if (first || t == 0) {
             flags |= kFirst;
             // units of this pair's first / last tile and of its head
-            const long long ftile = x - t, ltile = ftile + T - 1, pstart = ftile - kHead;
+            const long long ftile = x - t, ltile = ftile + T - 1, pstart = ftile - p.head;
             const int c = blockIdx.x;
             const int c0 = cta_of(ftile, W, N), c1 = cta_of(ltile, W, N);
             slot = (lo >= pstart) ? 2 * c : 2 * c + 1;   // first segment of this CTA?
@@ -276,7 +279,7 @@ struct TileWalker {
         ++x;
         if (++t == T) {                            // next pair: step over its head
             t = 0;
-            x += kHead;
+            x += p.head;
             if (++g == p.Hkv) {
                 g = 0;
                 if (x < end) {
