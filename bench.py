@@ -259,6 +259,18 @@ def oracle_sample_size(cfg, target_s=15.0, threads=None):
     return int(max(1, min(cfg.batch, n)))
 
 
+def workload_config(cfg, L):
+    """The `config` object both arms report for a workload."""
+    return {"workload": "%s: B=%d, L=%s, k=%d, %d/%d heads, D=%d, 64-token pages "
+                        "(shuffled=%s), draft %d sink + %d window"
+                        % (cfg.name, len(L), ("%d" % L[0]) if cfg.ctx_dist == "fixed" else
+                           "%s[%d,%d] (sum %d)" % (cfg.ctx_dist, cfg.ctx_lo, cfg.ctx_hi,
+                                                   int(L.sum())),
+                           cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim,
+                           cfg.paged_shuffle, cfg.n_sink, cfg.window),
+            "global_batch": int(len(L)), "seq_len": int(L.max()), "parallelism": "replicas"}
+
+
 def reference_arm(args, cfg):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -283,7 +295,7 @@ def reference_arm(args, cfg):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": per_step * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": cfg.name, "sample": sample},
+        "config": dict(workload_config(cfg, wl.sample_ctx_lens(cfg)), sample=sample),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -725,15 +737,9 @@ def spire_arm(args, cfg):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": "%s: B=%d, L=%s, k=%d, %d/%d heads, D=%d, 64-token pages "
-                               "(shuffled=%s), draft %d sink + %d window"
-                               % (cfg.name, B, ("%d" % L[0]) if cfg.ctx_dist == "fixed" else
-                                  "%s[%d,%d] (sum %d)" % (cfg.ctx_dist, cfg.ctx_lo, cfg.ctx_hi,
-                                                          int(L.sum())),
-                                  k, Hq, Hkv, D, cfg.paged_shuffle, cfg.n_sink, cfg.window),
-                   "global_batch": B, "seq_len": int(L.max()), "parallelism": "replicas",
-                   "l2": "flushed between steps (256 MB write); verify KV %.2f GB > L2"
-                         % (vb / 1e9)},
+        "config": dict(workload_config(cfg, L),
+                       l2="flushed between steps (256 MB write); verify KV %.2f GB > L2"
+                          % (vb / 1e9)),
         "roofline": {"kernel": "spire_verify_attention: attn_tc_kernel, launched with "
                                "programmatic dependent launch behind the one-CTA merge-counter "
                                "reset; CUDA events around the call",
