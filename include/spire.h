@@ -229,7 +229,7 @@ SPIRE_API spire_status spire_draft_sparse_attention(const void *q, const void *k
  * half-split pairs (d, d + D/2), angle p * rope_theta^(-2d/D)).
  */
 typedef struct spire_append_desc {
-    int32_t batch;            /* B >= 1 sequences, one new entry each */
+    int32_t batch;            /* B >= 0 sequences, one new entry each (0: nothing to do) */
     int32_t num_act;          /* n_layer + 1 activations mixed (1..16), x^0 = embedding */
     int32_t num_draft_layers; /* n_dl (1..16): memory vector, projection and cache per layer */
     int32_t d_model;          /* activation width, a multiple of 64 (64..65536) */
@@ -356,7 +356,7 @@ SPIRE_API size_t spire_verify_tokens_workspace_bytes(int32_t batch, int32_t k, i
  *   draft_tokens int32 [B, k]:     x_1..x_k (may be NULL if k = 0).
  *   u            fp32 [B, k]:      acceptance uniforms in [0, 1) (may be NULL if k = 0).
  *   e            fp32 [B, V]:      Exp(1) variates for the round's one draw.
- *   batch 1..65535, k 0..31, vocab V >= 1.
+ *   batch 0..65535 (0: nothing to do, any pointer may be NULL), k 0..31, vocab V >= 1.
  *   out_tokens   int32 [B, k+1]:   x_1..x_j, the drawn token, then -1.
  *   n_accepted   int32 [B]:        j.
  * Only the rows the round needs are read (p_{j+1}, q_{j+1}, E and k gathered

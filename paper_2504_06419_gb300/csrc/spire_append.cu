@@ -405,7 +405,7 @@ struct AppendPlan {
 
 bool plan_append(const spire_append_desc* d, AppendPlan* pl) {
     if (!d) return false;
-    if (d->batch < 1 || d->num_act < 1 || d->num_act > 16 || d->num_draft_layers < 1 ||
+    if (d->batch < 0 || d->num_act < 1 || d->num_act > 16 || d->num_draft_layers < 1 ||
         d->num_draft_layers > 16 || d->d_model < 64 || d->d_model > 65536 ||
         d->d_model % 64 != 0 || d->num_kv_heads < 1 || (d->head_dim != 64 && d->head_dim != 128) ||
         d->n_sink < 0 || d->window < 1 || !std::isfinite(d->rope_theta) || d->rope_theta < 0.f)
@@ -417,14 +417,19 @@ bool plan_append(const spire_append_desc* d, AppendPlan* pl) {
         (long long)d->num_draft_layers * d->batch > (1LL << 30))
         return false;
     pl->F = (int)F;
+    pl->mtiles = (int)(F / 128);
+    pl->kblocks = d->d_model / 64;
+    if (d->batch == 0) {           // nothing to do; the shape is still checked
+        pl->N = 16;
+        pl->ntb = 0;
+        return true;
+    }
     // one MMA covers the n_act activation tiles: n_act x N <= 256
     int nmax = (256 / d->num_act) / 16 * 16;
     if (nmax > kAppendMaxN) nmax = kAppendMaxN;
     const int nb = d->batch < nmax ? d->batch : nmax;
     pl->N = (nb + 15) / 16 * 16;
     pl->ntb = (d->batch + pl->N - 1) / pl->N;
-    pl->mtiles = (int)(F / 128);
-    pl->kblocks = d->d_model / 64;
     return true;
 }
 
@@ -449,12 +454,13 @@ spire_status spire_feedback_append(const void* x, const float* mix_w, const void
                                    const int32_t* pos, const spire_append_desc* desc, void* kv,
                                    void* workspace, size_t ws_bytes, void* stream) {
     AppendPlan pl;
-    if (!x || !mix_w || !w_kv || !pos || !kv || !workspace) return SPIRE_ERR_INVALID_ARG;
     if (!plan_append(desc, &pl)) {
-        if (desc && desc->head_dim != 64 && desc->head_dim != 128 && desc->batch >= 1)
+        if (desc && desc->head_dim != 64 && desc->head_dim != 128 && desc->batch >= 0)
             return SPIRE_ERR_UNSUPPORTED;
         return SPIRE_ERR_INVALID_ARG;
     }
+    if (desc->batch == 0) return SPIRE_OK;
+    if (!x || !mix_w || !w_kv || !pos || !kv || !workspace) return SPIRE_ERR_INVALID_ARG;
     if (!host_aligned(x, 16) || !host_aligned(w_kv, 16) || !host_aligned(kv, 16) ||
         !host_aligned(mix_w, 4) || !host_aligned(pos, 4) || !host_aligned(workspace, 256))
         return SPIRE_ERR_INVALID_ARG;

@@ -445,7 +445,7 @@ __global__ void __launch_bounds__(128) tokens_finalize_kernel(const TokParams p)
 }
 
 bool tok_shape_ok(int32_t B, int32_t k, int32_t V) {
-    return B >= 1 && B <= 65535 && k >= 0 && k <= kTokMaxK && V >= 1 && V <= (1 << 30) &&
+    return B >= 0 && B <= 65535 && k >= 0 && k <= kTokMaxK && V >= 1 && V <= (1 << 30) &&
            (long long)B * (k + 1) * V < (1LL << 40);
 }
 
@@ -474,12 +474,14 @@ spire_status spire_verify_tokens(const float* p, const float* q, const int32_t* 
                                  const float* u, const float* e, int32_t batch, int32_t k,
                                  int32_t vocab, int32_t* out_tokens, int32_t* n_accepted,
                                  void* workspace, size_t ws_bytes, void* stream) {
-    if (!p || !e || !out_tokens || !n_accepted || !workspace) return SPIRE_ERR_INVALID_ARG;
-    if (k > 0 && (!q || !draft_tokens || !u)) return SPIRE_ERR_INVALID_ARG;
     if (!tok_shape_ok(batch, k, vocab)) {
-        if (batch >= 1 && k > kTokMaxK && vocab >= 1) return SPIRE_ERR_UNSUPPORTED;
+        if (batch >= 0 && batch <= 65535 && k > kTokMaxK && vocab >= 1)
+            return SPIRE_ERR_UNSUPPORTED;
         return SPIRE_ERR_INVALID_ARG;
     }
+    if (batch == 0) return SPIRE_OK;              // nothing to do
+    if (!p || !e || !out_tokens || !n_accepted || !workspace) return SPIRE_ERR_INVALID_ARG;
+    if (k > 0 && (!q || !draft_tokens || !u)) return SPIRE_ERR_INVALID_ARG;
     if (!host_aligned(p, 4) || (q && !host_aligned(q, 4)) || !host_aligned(e, 4) ||
         (u && !host_aligned(u, 4)) || (draft_tokens && !host_aligned(draft_tokens, 4)) ||
         !host_aligned(out_tokens, 4) || !host_aligned(n_accepted, 4) ||

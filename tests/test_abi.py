@@ -140,10 +140,20 @@ def test_append_workspace_depends_only_on_shapes(spire):
     assert spire.spire_feedback_append_workspace_bytes(d) == n
     assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, batch=300)) == n
     assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, num_act=16, d_model=64)) == n
+    assert spire.spire_feedback_append_workspace_bytes(_adesc(spire, batch=0)) == n
+
+
+def test_append_empty_batch_is_a_no_op(spire):
+    # B = 0: the rest of the shape is still checked, nothing is read or launched
+    assert spire.spire_feedback_append(0, 0, 0, 0, _adesc(spire, batch=0), 0, 0, 0, 0) == 0
+    assert spire.spire_feedback_append(0, 0, 0, 0, _adesc(spire, batch=0, head_dim=96), 0, 0, 0,
+                                       0) == spire._lib.SPIRE_ERR_UNSUPPORTED
+    assert spire.spire_feedback_append(0, 0, 0, 0, _adesc(spire, batch=0, window=0), 0, 0, 0,
+                                       0) == spire._lib.SPIRE_ERR_INVALID_ARG
 
 
 @pytest.mark.parametrize("kw", [
-    dict(batch=0), dict(num_act=0), dict(num_act=17), dict(num_draft_layers=0),
+    dict(batch=-1), dict(num_act=0), dict(num_act=17), dict(num_draft_layers=0),
     dict(d_model=100), dict(d_model=0), dict(num_kv_heads=0), dict(head_dim=96),
     dict(n_sink=-1), dict(window=0), dict(rope_theta=-1.0), dict(rope_theta=float("inf")),
 ])
@@ -183,7 +193,8 @@ def test_tokens_workspace_and_host_checks(spire):
     # aligned), one 24-byte partial per 4096-entry chunk
     assert spire.spire_verify_tokens_workspace_bytes(64, 4, 128256) == 512 + 512 + 64 * 32 * 24
     assert spire.spire_verify_tokens_workspace_bytes(1, 0, 1) == 512 + 256 + 24
-    for bad in [(0, 4, 100), (1, -1, 100), (1, 32, 100), (1, 4, 0), (70000, 1, 10)]:
+    assert spire.spire_verify_tokens_workspace_bytes(0, 4, 100) == 512
+    for bad in [(-1, 4, 100), (1, -1, 100), (1, 32, 100), (1, 4, 0), (70000, 1, 10)]:
         assert spire.spire_verify_tokens_workspace_bytes(*bad) == 0
     good = 1 << 20
     ws = spire.spire_verify_tokens_workspace_bytes(8, 4, 1000)
@@ -198,7 +209,12 @@ def test_tokens_workspace_and_host_checks(spire):
     assert call(p=good + 2, vocab=1001) == E.SPIRE_ERR_INVALID_ARG
     assert call(ws_bytes=ws - 1) == E.SPIRE_ERR_WORKSPACE
     assert call(k=40) == E.SPIRE_ERR_UNSUPPORTED
-    assert call(batch=0) == E.SPIRE_ERR_INVALID_ARG
+    # B = 0: nothing to do, any pointer may be NULL; k and V are still checked
+    assert call(batch=0, p=0, q=0, draft_tokens=0, u=0, e=0, out_tokens=0, n_accepted=0,
+                workspace=0, ws_bytes=0) == E.SPIRE_OK
+    assert call(batch=0, k=40) == E.SPIRE_ERR_UNSUPPORTED
+    assert call(batch=0, vocab=0) == E.SPIRE_ERR_INVALID_ARG
+    assert call(batch=-1) == E.SPIRE_ERR_INVALID_ARG
 
 
 def test_magicdec_host_checks(spire):

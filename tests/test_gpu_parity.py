@@ -357,3 +357,28 @@ def test_split_plan_invariance(spire):
     done = parity.gpu_draft(spire, d1)
     rel, mx = parity.errors(dfull[0].cpu().numpy(), done[0].cpu().numpy())
     assert rel <= 1e-5 and mx <= 1e-5, (rel, mx)
+
+
+# ---------------------------------------------------------------- empty batches
+def test_every_call_accepts_an_empty_batch(spire):
+    """B = 0 is a no-op for every call: empty results, no device error."""
+    bf, f32, i32 = torch.bfloat16, torch.float32, torch.int32
+    q = torch.empty((0, 32, 128), dtype=bf, device=DEV)
+    kv = torch.empty((0, 2, 8, 528, 128), dtype=bf, device=DEV)
+    ctx = torch.empty((0,), dtype=i32, device=DEV)
+    assert spire.draft_attention(q, kv, ctx, 16, 512).shape == (0, 32, 128)
+    x = torch.empty((3, 0, 256), dtype=bf, device=DEV)
+    mix = torch.zeros((2, 3), dtype=f32, device=DEV)
+    w = torch.zeros((2, 2 * 2 * 64, 256), dtype=bf, device=DEV)
+    cache = torch.empty((2, 0, 2, 2, 7, 64), dtype=bf, device=DEV)
+    spire.feedback_append(x, mix, w, torch.empty((0,), dtype=i32, device=DEV), cache, 2, 5)
+    p = torch.empty((0, 5, 1000), dtype=f32, device=DEV)
+    toks, n_acc = spire.verify_tokens(p, torch.empty((0, 4, 1000), dtype=f32, device=DEV),
+                                      torch.empty((0, 4), dtype=i32, device=DEV),
+                                      torch.empty((0, 4), dtype=f32, device=DEV),
+                                      torch.empty((0, 1000), dtype=f32, device=DEV))
+    assert toks.shape == (0, 5) and n_acc.shape == (0,)
+    kc = torch.zeros((4, 8, 64, 128), dtype=bf, device=DEV)
+    bt = torch.empty((0, 1), dtype=i32, device=DEV)
+    assert spire.magicdec_attention(q, kc, kc, bt, ctx, 1, 64, 1e4).shape == (0, 32, 128)
+    torch.cuda.synchronize()
