@@ -49,3 +49,14 @@ def test_two_gloo_ranks_take_max_and_weak_scale():
 def test_single_rank_is_identity():
     assert bench.reduce_max([1.5, 2.5]) == [1.5, 2.5]
     assert bench.job_value(100, 1, 1.0) == 1e5
+
+
+def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
+    """Under torchrun the reference arm (the oracle on the host) runs and
+    prints on rank 0 alone; every other rank exits 0 without work."""
+    import argparse
+    import workloads as wl
+    monkeypatch.setenv("RANK", "1")
+    args = argparse.Namespace(steps=1, warmup=3, gpus=2)
+    assert bench.reference_arm(args, wl.CONFIGS["tiny"]) == 0
+    assert capsys.readouterr().out == ""
