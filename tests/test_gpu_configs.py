@@ -75,3 +75,32 @@ def test_draft_full_config(spire, name, window):
         parity.assert_close(out[sel].cpu().numpy(), ref, "draft %s w=%d step %d" % (name, w, j))
         del di, out
     torch.cuda.empty_cache()
+
+
+def test_magicdec_full_config(spire):
+    """The MagicDec draft step as the benchmark runs it: sink 1 + window 64
+    over the uniform 8K target cache (B = 64, 32/8 heads, D = 128, shuffled
+    pages), keys and query turned to cache positions (theta 1e4); the oracle
+    recomputes a sample of sequences from a compact copy of their pages."""
+    import oracle
+    cfg = wl.CONFIGS["uniform8k"]
+    L = wl.sample_ctx_lens(cfg)
+    vi = wl.make_verify(L, cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim,
+                        seed=cfg.seed, device=DEV, shuffle=cfg.paged_shuffle)
+    t = wl.draft_ctx_for_step(L, cfg.k, 0)
+    q = vi.q[:, 0].contiguous()
+    ctx = torch.as_tensor(t, dtype=torch.int32, device=DEV)
+    out = spire.magicdec_attention(q, vi.k_cache, vi.v_cache, vi.block_table, ctx, 1, 64, 1e4)
+    torch.cuda.synchronize()
+    seqs = _sample(t, 6, cfg.seed)
+    sub = parity.compact_verify(wl.VerifyInputs(q=vi.q, k_cache=vi.k_cache, v_cache=vi.v_cache,
+                                                block_table=vi.block_table, ctx_lens=ctx,
+                                                k=vi.k), seqs)
+    ref, n_bad = oracle.magicdec(wl.bf16_bits(sub.q[:, 0].contiguous()), wl.bf16_bits(sub.k_cache),
+                                 wl.bf16_bits(sub.v_cache), sub.block_table.cpu().numpy(),
+                                 sub.ctx_lens.cpu().numpy(), 1, 64, 1e4)
+    assert n_bad == 0
+    got = out[torch.tensor(seqs, device=DEV)].cpu().numpy()
+    parity.assert_close(got, ref, "magicdec uniform8k sequences %s" % seqs)
+    del vi, out
+    torch.cuda.empty_cache()
