@@ -11,9 +11,13 @@ synthetic N(0,1) bf16 tensors resident in HBM.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
                     [--impl spire|reference]
+    python bench.py --profile-call verify|decode|draft|append|tokens|magicdec
+                    [--config NAME] [--max-seqs N] [--warmup W] [--calls C]
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle
-on a bounded sample of the same workload instead.
+on a bounded sample of the same workload instead.  `--profile-call` makes only
+one kind of library call and exits (for small profiler captures); it prints no
+benchmark line.
 """
 from __future__ import annotations
 
@@ -195,6 +199,70 @@ def cta_balance(times):
             "busy_us_min": min(busy), "max_over_mean": max(busy) / mean if mean > 0 else None,
             "start_spread_us": (max(b for b, _ in times) - first) / 1e3,
             "span_us": (max(e for _, e in times) - first) / 1e3}
+
+
+def event_ms(call, n, flush, stream):
+    """Mean CUDA-event time (ms) of `call` over n launches, each after an L2
+    flush (a 256 MB write) outside the events, on `stream`."""
+    import torch
+    evs = []
+    for s in range(n):
+        flush.fill_(s & 0xff)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call()
+        b.record(stream)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+
+def verify_config_entry(spire, name, dev, stream, flush, args, hbm_peak, max_seqs=0, dist=None):
+    """Verification attention on another workload, timed as the headline
+    verify call: CUDA events around the C-ABI call, the 256 MB L2 flush
+    between launches, the same warm-up.  Frees its inputs before returning."""
+    import torch
+    cfg = wl.CONFIGS[name]
+    k, Hq, Hkv, D = cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+    L = wl.sample_ctx_lens(cfg)
+    if max_seqs:
+        L = L[:max_seqs]
+    vi = wl.make_verify(L, k, Hq, Hkv, D, seed=cfg.seed, device=dev, shuffle=cfg.paged_shuffle)
+    desc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+    ws = torch.empty(spire.spire_verify_workspace_bytes(desc, k), dtype=torch.uint8, device=dev)
+    out = torch.empty(vi.q.shape, dtype=torch.float32, device=dev)
+    sptr = stream.cuda_stream
+
+    def call():
+        st = spire.spire_verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table,
+                                          vi.ctx_lens, k, desc, out, ws, ws.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_verify_attention (%s)" % name)
+
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize(dev)
+    if spire.spire_get_device_error(ws, stream):
+        raise RuntimeError("device error word set by the %s verify call" % name)
+    n = max(1, min(args.steps, 100))
+    ms = reduce_max([event_ms(call, n, flush, stream)], dist, dev)[0]   # the slowest rank
+    flush.fill_(7)
+    call()
+    bal = cta_balance(spire.spire_get_cta_times(ws, ws.numel()))
+    vb = verify_bytes(L, k, Hq, Hkv, D)
+    gbs = vb / (ms * 1e-3) / 1e9
+    B = int(L.size)
+    entry = {"workload": workload_config(cfg, L)["workload"], "calls": n, "ms": ms,
+             "algorithmic_bytes": vb, "gbs": gbs, "frac": gbs / hbm_peak,
+             "frac_of_8TBs": gbs / HBM_NOMINAL_GBS,
+             "verify_tokens_per_s": B * (k + 1) / (ms * 1e-3),
+             "tflops": verify_flops(L, k, Hq, D) / (ms * 1e-3) / 1e12,
+             "rows_per_kv_head": (Hq // Hkv) * (k + 1),
+             "load_balance": bal,
+             "traffic": dram_traffic("verify:%s" % name)}
+    del vi, ws, out
+    torch.cuda.empty_cache()
+    return entry
 
 
 def job_value(tokens_per_rank, world, step_ms):
@@ -712,6 +780,16 @@ def spire_arm(args, cfg):
         del sdi, sw_ctx, sw_ws, sw_out
         torch.cuda.empty_cache()
 
+    # ---- verification on the other two verify workloads, the ragged serving mix
+    # (B = 64, k = 4, L log-uniform in [1024, 131072]) and the large batch with
+    # deeper speculation (B = 256, k = 8, 64/8 heads), timed as the headline call
+    verify_configs = {}
+    for name in ("ragged", "big"):
+        if name == cfg.name:
+            continue
+        verify_configs[name] = verify_config_entry(spire, name, dev, stream, flush, args,
+                                                   hbm_peak, dist=dist)
+
     if rank != 0:
         if dist is not None:
             dist.barrier()
@@ -782,6 +860,7 @@ def spire_arm(args, cfg):
                        "gbs": tb / (tok_ms * 1e-3) / 1e9,
                        "frac": tb / (tok_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
                        "mean_accepted": float(n_acc_h.mean()), "launches": 3},
+                   "verify_configs": verify_configs,
                    "draft_sweep": {
                        "what": "B=%d, t log-uniform [4096, 262144], %d draft steps per round on "
                                "one bounded cache per window, each step's cache streamed from "
@@ -806,6 +885,102 @@ def spire_arm(args, cfg):
     return 0
 
 
+def profile_call(args, cfg):
+    """One library call, for profiler captures: allocate only that call's inputs
+    (the workload, cut to --max-seqs sequences when given), make --warmup calls
+    and then --calls more, each after the 256 MB L2 flush, and exit.  Prints a
+    one-line summary, never a benchmark line (times taken under a profiler are
+    not measurements)."""
+    import torch
+
+    import paper_2504_06419_gb300 as spire
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    k, Hq, Hkv, D = cfg.k, cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+    L = wl.sample_ctx_lens(cfg)
+    if args.max_seqs:
+        L = L[:args.max_seqs]
+    B = int(L.size)
+    what = args.profile_call
+    ws = None
+    if what in ("verify", "decode", "magicdec"):
+        vi = wl.make_verify(L, k, Hq, Hkv, D, seed=cfg.seed, device=dev, shuffle=cfg.paged_shuffle)
+        desc = spire.verify_desc(vi.q, vi.k_cache, vi.block_table)
+        if what == "magicdec":
+            t = torch.from_numpy(wl.draft_ctx_for_step(L, k, 0)).to(dev)
+            q = vi.q[:, 0].contiguous()
+            out = torch.empty(q.shape, dtype=torch.float32, device=dev)
+            ws = torch.empty(spire.spire_magicdec_workspace_bytes(desc, 1, 64), dtype=torch.uint8,
+                             device=dev)
+
+            def call():
+                return spire.spire_magicdec_attention(q, vi.k_cache, vi.v_cache, vi.block_table, t,
+                                                      1, 64, 10000.0, desc, out, ws, ws.numel(),
+                                                      sptr)
+        else:
+            kk = k if what == "verify" else 0
+            q = vi.q if kk == k else vi.q[:, :1].contiguous()
+            ctx = vi.ctx_lens if kk == k else (vi.ctx_lens - k).contiguous()
+            out = torch.empty(q.shape, dtype=torch.float32, device=dev)
+            ws = torch.empty(spire.spire_verify_workspace_bytes(desc, kk), dtype=torch.uint8,
+                             device=dev)
+
+            def call():
+                return spire.spire_verify_attention(q, vi.k_cache, vi.v_cache, vi.block_table, ctx,
+                                                    kk, desc, out, ws, ws.numel(), sptr)
+    elif what == "draft":
+        di = wl.make_draft(wl.draft_ctx_for_step(L, k, 0), Hq, Hkv, D, cfg.n_sink, cfg.window,
+                           seed=cfg.seed + 17, device=dev)
+        desc = spire.draft_desc(di.q, di.kv)
+        ws = torch.empty(spire.spire_draft_workspace_bytes(desc, cfg.n_sink, cfg.window),
+                         dtype=torch.uint8, device=dev)
+        out = torch.empty(di.q.shape, dtype=torch.float32, device=dev)
+
+        def call():
+            return spire.spire_draft_sparse_attention(di.q, di.kv, di.ctx_lens, cfg.n_sink,
+                                                      cfg.window, desc, out, ws, ws.numel(), sptr)
+    elif what == "append":
+        n_dl, n_act, d_model = 2, 3, Hq * D
+        ai = wl.make_append(wl.draft_ctx_for_step(L, k, 0), n_act, n_dl, d_model, Hkv, D,
+                            cfg.n_sink, cfg.window, seed=cfg.seed + 101, device=dev)
+        adesc = spire.make_append_desc(B, n_act, n_dl, d_model, Hkv, D, cfg.n_sink, cfg.window,
+                                       10000.0)
+        ws = torch.empty(spire.spire_feedback_append_workspace_bytes(adesc), dtype=torch.uint8,
+                         device=dev)
+
+        def call():
+            return spire.spire_feedback_append(ai.x, ai.mix_w, ai.w_kv, ai.pos, adesc, ai.kv, ws,
+                                               ws.numel(), sptr)
+    elif what == "tokens":
+        V_tok = 128256
+        ti = wl.make_tokens(B, k, V_tok, seed=cfg.seed + 202, device=dev)
+        ws = torch.empty(spire.spire_verify_tokens_workspace_bytes(B, k, V_tok), dtype=torch.uint8,
+                         device=dev)
+        tok_out = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+        tok_acc = torch.empty((B,), dtype=torch.int32, device=dev)
+
+        def call():
+            return spire.spire_verify_tokens(ti.p, ti.q, ti.x, ti.u, ti.e, B, k, V_tok, tok_out,
+                                             tok_acc, ws, ws.numel(), sptr)
+    else:
+        raise ValueError(what)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    n = args.warmup + args.calls
+    for s in range(n):
+        flush.fill_(s & 0xff)
+        st = call()
+        if st:
+            raise spire.SpireError(st, what)
+    torch.cuda.synchronize(dev)
+    err = spire.spire_get_device_error(ws, stream) if what != "tokens" else 0
+    print("profile-call %s on %s (%d sequences): %d calls (%d warm-up), device error word %d"
+          % (what, cfg.name, B, n, args.warmup, err), flush=True)
+    return 1 if err else 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -817,10 +992,18 @@ def main():
     ap.add_argument("--max-seqs", type=int, default=0,
                     help="use only the first N sequences of the workload (small profiling "
                          "captures; not a benchmark configuration)")
+    ap.add_argument("--profile-call", default=None,
+                    choices=["verify", "decode", "draft", "append", "tokens", "magicdec"],
+                    help="make only this library call (--warmup + --calls times, each after "
+                         "the L2 flush) and exit: small profiler captures, never a benchmark")
+    ap.add_argument("--calls", type=int, default=2,
+                    help="calls after the warm-up in --profile-call mode")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     cfg = wl.CONFIGS[args.config]
+    if args.profile_call:
+        return profile_call(args, cfg)
     if args.impl == "reference":
         return reference_arm(args, cfg)
     return spire_arm(args, cfg)

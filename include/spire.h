@@ -158,12 +158,17 @@ SPIRE_API spire_status spire_verify_attention(const void *q, const void *k_cache
  * workspace: its scratch (split partials, arrival counters, error words) is
  * one file-scope device array of 32 MiB, reserved on every GPU that loads
  * libspire until the process exits.  Nothing is allocated by the call.
- *   - A shape whose workspace (spire_verify_workspace_bytes) exceeds 32 MiB
- *     returns SPIRE_ERR_WORKSPACE; at head_dim 128 that allows up to about 60
- *     query rows per KV head ((Hq/Hkv)*(k+1)).  Invalid shapes return the same
- *     status as spire_verify_attention.
+ *   - A valid, non-empty shape whose workspace (spire_verify_workspace_bytes)
+ *     exceeds 32 MiB returns SPIRE_ERR_WORKSPACE; at head_dim 128 that allows
+ *     up to about 60 query rows per KV head ((Hq/Hkv)*(k+1)).  Every other
+ *     case returns what spire_verify_attention returns: an empty batch is a
+ *     no-op (SPIRE_OK), an unsupported page size SPIRE_ERR_UNSUPPORTED, null
+ *     or misaligned pointers SPIRE_ERR_INVALID_ARG.
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.  The address is looked up again when the
+ *     device's context has changed since (after cudaDeviceReset, for
+ *     example), so such a call, too, belongs outside a capture.
  *   - All calls share the one array: calls that may overlap on the GPU (on
  *     different streams, or from different threads) race and must not be
  *     issued.  The array keeps the last call's contents; each call clears what
@@ -375,9 +380,28 @@ SPIRE_API spire_status spire_verify_tokens(const float *p, const float *q,
 
 /*
  * spire_draft_slot -- slot of logical memory position p >= 0 in the bounded
- * draft cache: p if p < n_sink, else n_sink + (p - n_sink) mod window.
- * Returns -1 for p < 0, n_sink < 0 or window < 1.  Host function.
+ * draft cache (Section 3.1: attention sinks kept, a sliding window over the
+ * rest, so the cache never grows): p if p < n_sink, else
+ * n_sink + (p - n_sink) mod window.  Returns -1 for p < 0, n_sink < 0 or
+ * window < 1.  Exported host function (for callers through an FFI).
+ *
+ * spire_draft_slot_inline is the same function, defined here for host code
+ * and for CUDA device code (compiled by nvcc it is __host__ __device__).  It
+ * is the one definition: the exported function and the kernel that writes
+ * new entries into the cache (spire_feedback_append) both use it.
  */
+#if defined(__CUDACC__)
+#define SPIRE_HOST_DEVICE __host__ __device__
+#else
+#define SPIRE_HOST_DEVICE
+#endif
+static inline SPIRE_HOST_DEVICE int64_t spire_draft_slot_inline(int64_t pos, int32_t n_sink,
+                                                               int32_t window) {
+    if (pos < 0 || n_sink < 0 || window < 1) return -1;
+    if (pos < n_sink) return pos;
+    return n_sink + (pos - n_sink) % window;
+}
+
 SPIRE_API int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
 
 /*

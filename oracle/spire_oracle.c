@@ -38,7 +38,7 @@
  *                         window over the target's own paged cache, positions
  *                         inside the reduced cache (Section 3.1 footnote).
  *
- * Readings of points the paper leaves open (all listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - scores are softmax_scale * <q, k>; the workloads pre-scale q, scale = 1;
  *   - verify ctx_lens[b] = L counts the cache entries including the k+1 block
  *     tokens; block row i (0..k) sees keys j < L - k + i;

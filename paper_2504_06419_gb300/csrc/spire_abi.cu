@@ -907,9 +907,7 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
 }
 
 int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {
-    if (pos < 0 || n_sink < 0 || window < 1) return -1;
-    if (pos < n_sink) return pos;
-    return n_sink + (pos - n_sink) % window;
+    return spire_draft_slot_inline(pos, n_sink, window);
 }
 
 spire_status spire_get_device_error(const void* workspace, int32_t* code_out, void* stream) {
@@ -982,21 +980,58 @@ constexpr size_t kStaticWsBytes = size_t(32) << 20;   // 32 MiB
 
 static __device__ __align__(256) unsigned char g_static_ws[kStaticWsBytes];
 
-// Device address of g_static_ws on the current device, looked up once per
-// device (cudaGetSymbolAddress, which allocates nothing).
+// Unique id of the calling thread's current context, or 0 when there is none
+// (or the driver lacks cuCtxGetId).  A context created after cudaDeviceReset
+// gets a new id even where its handle value repeats, so a device address
+// cached for an older context is never reused.
+unsigned long long current_ctx_id() {
+    using GetCurrent = CUresult (*)(CUcontext*);
+    using GetId = CUresult (*)(CUcontext, unsigned long long*);
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(p);
+    });
+    if (!get_current || !get_id) return 0;
+    CUcontext c = nullptr;
+    if (get_current(&c) != CUDA_SUCCESS || !c) return 0;
+    unsigned long long id = 0;
+    return get_id(c, &id) == CUDA_SUCCESS ? id : 0;
+}
+
+// Device address of g_static_ws on the current device, looked up
+// (cudaGetSymbolAddress, which allocates nothing) on the first call for each
+// device and again whenever the device's context has changed since.
 spire_status static_ws_address(void** out) {
     static std::mutex mu;
     static void* addr[64] = {};
+    static unsigned long long ctx[64] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return SPIRE_ERR_CUDA;
     std::lock_guard<std::mutex> g(mu);
-    if (dev >= 0 && dev < 64 && addr[dev]) {
+    const bool slot = dev >= 0 && dev < 64;
+    const unsigned long long id = current_ctx_id();
+    if (slot && addr[dev] && id != 0 && ctx[dev] == id) {
         *out = addr[dev];
         return SPIRE_OK;
     }
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || !p) return SPIRE_ERR_CUDA;
-    if (dev >= 0 && dev < 64) addr[dev] = p;
+    if (slot) {
+        addr[dev] = p;
+        ctx[dev] = current_ctx_id();   // the lookup made the primary context current if none was
+    }
     *out = p;
     return SPIRE_OK;
 }
@@ -1009,11 +1044,14 @@ extern "C" spire_status spire_verify_attention_noalloc(const void* q, const void
                                                        const int32_t* ctx_lens, int32_t k,
                                                        const spire_attn_desc* desc, float* out,
                                                        void* stream) {
-    const size_t need = spire_verify_workspace_bytes(desc, k);
-    if (need == 0)   // invalid shapes: report them exactly as the workspace entry point does
+    // Invalid descriptors have no workspace size: report them exactly as the
+    // workspace entry point does.  Otherwise its ordered checks see the static
+    // array, so a valid, non-empty shape that needs more than it holds is the
+    // only one that gets SPIRE_ERR_WORKSPACE (an empty batch is a no-op, an
+    // unsupported page size SPIRE_ERR_UNSUPPORTED, as there).
+    if (spire_verify_workspace_bytes(desc, k) == 0)
         return spire_verify_attention(q, k_cache, v_cache, block_table, ctx_lens, k, desc, out,
                                       nullptr, 0, stream);
-    if (need > kStaticWsBytes) return SPIRE_ERR_WORKSPACE;
     void* ws = nullptr;
     const spire_status st = static_ws_address(&ws);
     if (st != SPIRE_OK) return st;

@@ -267,10 +267,8 @@ __global__ void __launch_bounds__(kAppendThreads, 1)
             const int b = nt * N + j0 + e;
             const int pos = b < p.B ? p.pos[b] : INT_MIN;
             spos[e] = pos;
-            sslot[e] = pos == INT_MIN ? INT_MIN
-                       : pos < 0      ? -1
-                       : pos < p.n_sink ? pos
-                                        : p.n_sink + (pos - p.n_sink) % p.window;
+            sslot[e] = pos == INT_MIN ? INT_MIN   // no sequence: nothing to store
+                                      : (int)spire_draft_slot_inline(pos, p.n_sink, p.window);
         }
         named_bar_sync(1, 256);                  // amix is written
         if (!mbar_wait(bar_acc, 0)) err |= kErrTimeout;

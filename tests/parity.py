@@ -2,7 +2,11 @@
 run the oracle on the very same inputs, and compare.
 
 Tolerance (per call, over the whole compared output): max |gpu - oracle| <= 1e-2
-and ||gpu - oracle||_2 / ||oracle||_2 <= 1e-3.
+and ||gpu - oracle||_2 / ||oracle||_2 <= 1e-3.  Also per output row (one
+(sequence, block row, query head) vector of head_dim values): the row's
+relative L2 error <= 1e-3, so that a wrong row of a long sequence, whose
+outputs are small (|o| ~ 1/sqrt(L) for flat logits), cannot hide behind the
+larger outputs of short sequences in the whole-tensor norm.
 """
 from __future__ import annotations
 
@@ -14,6 +18,16 @@ import workloads as wl
 
 MAX_ABS = 1e-2
 REL_L2 = 1e-3
+# Per-row bound where an attention operand is itself computed and rounded to
+# bf16 before the attention (MagicDec's keys and query turned to cache
+# positions; a draft step over entries the feedback append just wrote).  The
+# kernel computes such a value in fp32 and the oracle in fp64, so a value that
+# lies next to a bf16 rounding boundary can round to the neighbouring bf16
+# number on one side: one element moves by one bf16 unit (2^-8 of it), one
+# score by up to |q_d| 2^-8 |k_d| (about 1e-2 for the largest N(0,1) entries),
+# and a row that a few keys dominate by up to about that much, relatively.
+# Such rows are held to 1e-2; the whole-tensor gates above stay as they are.
+ROW_REL_REROUNDED = 1e-2
 
 
 def errors(got: np.ndarray, ref: np.ndarray):
@@ -27,10 +41,31 @@ def errors(got: np.ndarray, ref: np.ndarray):
     return rel, float(np.abs(diff).max())
 
 
-def assert_close(got, ref, what=""):
+def row_errors(got: np.ndarray, ref: np.ndarray):
+    """Relative L2 error of every row (the last axis) and the worst row.
+    Returns (rel per row, index tuple of the worst row, its rel).  A row whose
+    reference is exactly zero counts its absolute L2 error instead."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape
+    if got.size == 0:
+        return np.zeros(got.shape[:-1]), (), 0.0
+    num = np.linalg.norm(got - ref, axis=-1)
+    den = np.linalg.norm(ref, axis=-1)
+    rel = np.where(den > 0, num / np.where(den > 0, den, 1.0), num)
+    worst = np.unravel_index(int(np.argmax(rel)), rel.shape)
+    return rel, tuple(int(i) for i in worst), float(rel[worst])
+
+
+def assert_close(got, ref, what="", row_rel=REL_L2):
+    """Whole-tensor gates (rel L2 <= 1e-3, max abs <= 1e-2) and the per-row
+    gate row_rel (1e-3; ROW_REL_REROUNDED where operands were re-rounded)."""
     assert np.all(np.isfinite(got)), "%s: non-finite GPU output" % what
     rel, mx = errors(got, ref)
     assert rel <= REL_L2 and mx <= MAX_ABS, "%s: rel_l2=%.3g max_abs=%.3g" % (what, rel, mx)
+    _, worst, wrel = row_errors(got, ref)
+    assert wrel <= row_rel, "%s: row %s has rel_l2=%.3g (whole tensor %.3g)" % (
+        what, worst, wrel, rel)
     return rel, mx
 
 

@@ -161,7 +161,7 @@ def test_append_then_draft_attention():
     attend with t + 1 visible entries (the new entry included); compared with
     the oracle's append followed by its draft attention."""
     import paper_2504_06419_gb300 as spire
-    from parity import assert_close
+    from parity import ROW_REL_REROUNDED, assert_close
     t = np.array([0, 5, 20, 47, 300], dtype=np.int32)
     n_sink, window, Hq, Hkv, D = 4, 16, 8, 2, 128
     ai = wl.make_append(t, 3, 1, 256, Hkv, D, n_sink, window, seed=31, device="cuda")
@@ -175,4 +175,4 @@ def test_append_then_draft_attention():
     # the oracle attends over its own appended cache
     ref, n_bad = oracle.draft_ring(wl.bf16_bits(q), want_kv[0], t + 1, n_sink, window)
     assert n_bad == 0
-    assert_close(out.cpu().double().numpy(), ref, "append + draft")
+    assert_close(out.cpu().double().numpy(), ref, "append + draft", row_rel=ROW_REL_REROUNDED)

@@ -6,7 +6,7 @@ import torch
 
 import oracle
 import workloads as wl
-from parity import assert_close
+from parity import ROW_REL_REROUNDED, assert_close
 
 pytestmark = pytest.mark.gpu
 
@@ -47,7 +47,7 @@ def test_magicdec_matches_oracle(case):
     _, L, Hq, Hkv, D, n_sink, window, theta = case
     got, ref, err, n_bad = _run(np.array(L), Hq, Hkv, D, n_sink, window, theta, seed=len(L) + D)
     assert n_bad == 0 and err == 0
-    assert_close(got, ref, "magicdec")
+    assert_close(got, ref, "magicdec", row_rel=ROW_REL_REROUNDED)
 
 
 def test_magicdec_invalid_sequences_are_nan():
@@ -60,4 +60,4 @@ def test_magicdec_invalid_sequences_are_nan():
     got, ref, err, n_bad = _run(L, 4, 1, 64, 1, 16, 10000.0, seed=3, edit=edit)
     assert n_bad == 3 and err == 1       # SPIRE_DEVERR_CTX_LEN
     assert np.all(np.isnan(got[:3])) and np.all(np.isfinite(got[3]))
-    assert_close(got[3:], ref[3:], "magicdec valid row")
+    assert_close(got[3:], ref[3:], "magicdec valid row", row_rel=ROW_REL_REROUNDED)
