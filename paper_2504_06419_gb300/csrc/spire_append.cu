@@ -469,6 +469,9 @@ spire_status spire_feedback_append(const void* x, const float* mix_w, const void
 
     const int B = desc->batch, n_dl = desc->num_draft_layers, n_act = desc->num_act;
     const int NA = n_act * pl.N, TS = (NA + 31) / 32 * 32;
+    // One MMA's N is NA, and an activation stage holds exactly NA rows: both
+    // come from this plan, within what a kind::f16 MMA with M = 128 accepts.
+    if (NA < 16 || NA > 256 || NA % 16 != 0) return SPIRE_ERR_UNSUPPORTED;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return SPIRE_ERR_CUDA;
     const long long tiles1 = (long long)n_dl * pl.mtiles * pl.ntb;
