@@ -201,13 +201,32 @@ def cta_balance(times):
             "span_us": (max(e for _, e in times) - first) / 1e3}
 
 
-def event_ms(call, n, flush, stream):
-    """Mean CUDA-event time (ms) of `call` over n launches, each after an L2
-    flush (a 256 MB write) outside the events, on `stream`."""
+class L2Flush:
+    """Empties L2 of every input between timed launches: a 256 MB write (twice
+    the 129 MB L2), then a read of that buffer, so that L2 holds only the
+    buffer's clean lines.  A write alone leaves L2 full of dirty lines whose
+    write-back the next timed kernel would pay (about 16 us for a verify call
+    on GB300), which no step of a serving loop, where L2 mostly holds lines
+    read by the previous kernels, would see."""
+
+    def __init__(self, dev):
+        import torch
+        self.buf = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+        self.words = self.buf.view(torch.int64)
+
+    def __call__(self, s, write_only=False):
+        self.buf.fill_(s & 0xff)
+        if not write_only:
+            self.words.amax()
+
+
+def event_ms(call, n, flush, stream, write_only=False):
+    """Mean CUDA-event time (ms) of `call` over n launches, each after the L2
+    flush outside the events, on `stream`."""
     import torch
     evs = []
     for s in range(n):
-        flush.fill_(s & 0xff)
+        flush(s, write_only)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         call()
@@ -246,7 +265,7 @@ def verify_config_entry(spire, name, dev, stream, flush, args, hbm_peak, max_seq
         raise RuntimeError("device error word set by the %s verify call" % name)
     n = max(1, min(args.steps, 100))
     ms = reduce_max([event_ms(call, n, flush, stream)], dist, dev)[0]   # the slowest rank
-    flush.fill_(7)
+    flush(7)
     call()
     bal = cta_balance(spire.spire_get_cta_times(ws, ws.numel()))
     vb = verify_bytes(L, k, Hq, Hkv, D)
@@ -424,7 +443,7 @@ def spire_arm(args, cfg):
         if st:
             raise spire.SpireError(st, "spire_draft_sparse_attention")
 
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # 2x the 129 MB L2
+    flush = L2Flush(dev)
 
     def barrier():
         if dist is not None:
@@ -446,7 +465,7 @@ def spire_arm(args, cfg):
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(k + 2)] for _ in range(n_detail)]
     barrier()
     for s in range(n_detail):
-        flush.fill_(s & 0xff)          # L2 flush between steps, outside the events
+        flush(s & 0xff)          # L2 flush between steps, outside the events
         e = ev[s]
         e[0].record(stream)
         call_verify()
@@ -456,6 +475,8 @@ def spire_arm(args, cfg):
             e[2 + j].record(stream)
     barrier()
     eager_ms = statistics.mean(e[0].elapsed_time(e[-1]) for e in ev)
+    # the verify call after a write-only flush (L2 left full of dirty lines), for comparison
+    v_ms_dirty = event_ms(call_verify, n_detail, flush, stream, write_only=True)
     v_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
     d_ms = statistics.mean(sum(e[1 + j].elapsed_time(e[2 + j]) for j in range(k)) for e in ev)
 
@@ -475,7 +496,7 @@ def spire_arm(args, cfg):
         call_decode()
     dec_ev = []
     for s in range(n_detail):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         call_decode()
@@ -509,7 +530,7 @@ def spire_arm(args, cfg):
     barrier()
     t0 = time.time()
     for s in range(args.steps):
-        flush.fill_(s & 0xff)          # L2 flush between steps, outside the events
+        flush(s & 0xff)          # L2 flush between steps, outside the events
         gev[s][0].record(stream)
         graph.replay()
         gev[s][1].record(stream)
@@ -517,7 +538,8 @@ def spire_arm(args, cfg):
     t1 = time.time()
     clocks = sampler.stop(t0, t1)
     ms = statistics.mean(e[0].elapsed_time(e[1]) for e in gev)
-    ms, eager_ms, v_ms, d_ms, dec_ms = reduce_max([ms, eager_ms, v_ms, d_ms, dec_ms], dist, dev)
+    ms, eager_ms, v_ms, d_ms, dec_ms, v_ms_dirty = reduce_max(
+        [ms, eager_ms, v_ms, d_ms, dec_ms, v_ms_dirty], dist, dev)
     del graph
 
     B = int(L.size)
@@ -578,7 +600,7 @@ def spire_arm(args, cfg):
     e2e_steps = max(1, min(args.steps, 200))
     e2e_ms = []
     for s in range(e2e_steps):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         e2e_step()
@@ -588,10 +610,10 @@ def spire_arm(args, cfg):
     e2e_val = job_value(tokens, world, reduce_max([statistics.mean(e2e_ms)], dist, dev)[0])
 
     # ---- load balance: per-SM busy time of one verify and one draft call
-    flush.fill_(1)
+    flush(1)
     call_verify()
     bal_v = cta_balance(spire.spire_get_cta_times(ws_v, ws_v.numel()))
-    flush.fill_(2)
+    flush(2)
     call_draft(0)
     bal_d = cta_balance(spire.spire_get_cta_times(ws_d, ws_d.numel()))
 
@@ -632,7 +654,7 @@ def spire_arm(args, cfg):
     a_steps = max(1, min(args.steps, 200))
     a_ev = []
     for s in range(a_steps):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         call_append(s % k)
@@ -652,7 +674,7 @@ def spire_arm(args, cfg):
     torch.cuda.synchronize(dev)
     p_ev = []
     for s in range(a_steps):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         pgraph.replay()
@@ -685,7 +707,7 @@ def spire_arm(args, cfg):
     torch.cuda.synchronize(dev)
     t_ev = []
     for s in range(a_steps):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         call_tokens()
@@ -716,7 +738,7 @@ def spire_arm(args, cfg):
     torch.cuda.synchronize(dev)
     md_ev = []
     for s in range(a_steps):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         call_magicdec(s % k)
@@ -761,7 +783,7 @@ def spire_arm(args, cfg):
         sw_ev = []
         for s in range(max(1, min(args.steps, 50))):
             for j in range(sw_k):
-                flush.fill_((s + j) & 0xff)     # each step streams its cache from HBM
+                flush((s + j) & 0xff)     # each step streams its cache from HBM
                 a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 a.record(stream)
                 call_sweep(j)
@@ -790,6 +812,29 @@ def spire_arm(args, cfg):
         verify_configs[name] = verify_config_entry(spire, name, dev, stream, flush, args,
                                                    hbm_peak, dist=dist)
 
+    # ---- the floor of a single launch that reads a call's algorithmic bytes:
+    # spire_stream_read streams that many bytes with the attention kernels' copy
+    # machinery and computes nothing (same flush, same events)
+    floor_buf = torch.empty(int(max(vb, db // k, ab, tb, md_bytes)) + 16, dtype=torch.uint8,
+                            device=dev)
+
+    def floor_us(nbytes):
+        nb = int(nbytes) // 16 * 16
+
+        def call():
+            st = spire.spire_stream_read(floor_buf, nb, sptr)
+            if st:
+                raise spire.SpireError(st, "spire_stream_read")
+
+        for _ in range(max(3, args.warmup)):
+            call()
+        return reduce_max([event_ms(call, max(1, min(args.steps, 100)), flush, stream)], dist,
+                          dev)[0] * 1e3
+
+    floors = {"verify": floor_us(vb), "draft_step": floor_us(db // k), "append": floor_us(ab),
+              "tokens": floor_us(tb), "magicdec": floor_us(md_bytes)}
+    del floor_buf
+
     if rank != 0:
         if dist is not None:
             dist.barrier()
@@ -816,8 +861,9 @@ def spire_arm(args, cfg):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": dict(workload_config(cfg, L),
-                       l2="flushed between steps (256 MB write); verify KV %.2f GB > L2"
-                          % (vb / 1e9)),
+                       l2="flushed between steps (a 256 MB write, then a read of that buffer: "
+                          "L2 holds none of the inputs and no dirty lines); verify KV %.2f GB "
+                          "> L2" % (vb / 1e9)),
         "roofline": {"kernel": "spire_verify_attention: attn_tc_kernel, launched with "
                                "programmatic dependent launch behind the one-CTA merge-counter "
                                "reset; CUDA events around the call",
@@ -828,6 +874,15 @@ def spire_arm(args, cfg):
         "detail": {"round": "one CUDA graph per step (verify + %d draft calls); "
                              "eager launches: %.4f ms per step" % (k, eager_ms),
                    "verify_ms": v_ms, "draft_ms_total": d_ms, "verify_gbs": v_gbs,
+                   "verify_ms_after_write_only_flush": v_ms_dirty,
+                   "stream_floor": {
+                       "what": "spire_stream_read: one launch that reads the call's algorithmic "
+                               "bytes with the same bulk-copy ring and computes nothing, timed "
+                               "like the calls (us); floor_over_us = floor / the call's time",
+                       "verify_us": floors["verify"],
+                       "verify_floor_over_us": floors["verify"] / (v_ms * 1e3),
+                       "draft_step_us": floors["draft_step"],
+                       "draft_step_floor_over_us": floors["draft_step"] / (d_ms / k * 1e3)},
                    "draft_gbs": d_gbs, "draft_bytes_per_round": db,
                    "verify_tokens_per_s": world * tokens / (v_ms * 1e-3),
                    "draft_tokens_per_s": world * B * k / (d_ms * 1e-3),
@@ -839,6 +894,8 @@ def spire_arm(args, cfg):
                        "us": app_ms * 1e3, "algorithmic_bytes": ab,
                        "gbs": ab / (app_ms * 1e-3) / 1e9,
                        "frac": ab / (app_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
+                       "floor_us": floors["append"],
+                       "floor_over_us": floors["append"] / (app_ms * 1e3),
                        "launches": 1},
                    "perf_model": perf_model_detail(L, k, Hq, Hkv, D, S, v_ms, d_ms, dec_ms),
                    "load_balance": {
@@ -853,12 +910,16 @@ def spire_arm(args, cfg):
                                % (md_sink, md_win),
                        "us": md_ms * 1e3, "algorithmic_bytes": md_bytes,
                        "gbs": md_bytes / (md_ms * 1e-3) / 1e9,
+                       "floor_us": floors["magicdec"],
+                       "floor_over_us": floors["magicdec"] / (md_ms * 1e3),
                        "spire_draft_step_us": d_ms / k * 1e3},
                    "verify_tokens": {
                        "shape": "B=%d, k=%d, vocabulary %d (fp32 distributions)" % (B, k, V_tok),
                        "us": tok_ms * 1e3, "algorithmic_bytes": tb,
                        "gbs": tb / (tok_ms * 1e-3) / 1e9,
                        "frac": tb / (tok_ms * 1e-3) / 1e9 / hbm_peak, "bound": "hbm",
+                       "floor_us": floors["tokens"],
+                       "floor_over_us": floors["tokens"] / (tok_ms * 1e3),
                        "mean_accepted": float(n_acc_h.mean()), "launches": 3},
                    "verify_configs": verify_configs,
                    "draft_sweep": {
@@ -967,10 +1028,10 @@ def profile_call(args, cfg):
                                              tok_acc, ws, ws.numel(), sptr)
     else:
         raise ValueError(what)
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    flush = L2Flush(dev)
     n = args.warmup + args.calls
     for s in range(n):
-        flush.fill_(s & 0xff)
+        flush(s & 0xff)
         st = call()
         if st:
             raise spire.SpireError(st, what)

@@ -379,6 +379,21 @@ SPIRE_API spire_status spire_verify_tokens(const float *p, const float *q,
                                            size_t ws_bytes, void *stream);
 
 /*
+ * spire_stream_read -- a measurement helper; the paper has no counterpart.
+ * One kernel launch that reads `bytes` of device memory at `src` once and
+ * computes nothing: one CTA per SM streams a contiguous run of 16 KB chunks
+ * through a ring of shared-memory stages with bulk async copies, as the
+ * attention kernels stream their K/V tiles.  Its time is the floor of any
+ * single launch of this library that must read that many bytes (launch,
+ * first-byte latency and the stream), against which calls that move tens of
+ * MB -- a draft step, the feedback append, token verification -- are
+ * compared.  src must be 16-byte aligned and bytes a multiple of 16
+ * (SPIRE_ERR_INVALID_ARG otherwise); bytes = 0 is a no-op.  Nothing is
+ * written; asynchronous on `stream`.
+ */
+SPIRE_API spire_status spire_stream_read(const void *src, size_t bytes, void *stream);
+
+/*
  * spire_draft_slot -- slot of logical memory position p >= 0 in the bounded
  * draft cache (Section 3.1: attention sinks kept, a sliding window over the
  * rest, so the cache never grows): p if p < n_sink, else

@@ -44,6 +44,7 @@ EXPORTED = (
     "spire_draft_slot",
     "spire_get_device_error",
     "spire_get_cta_times",
+    "spire_stream_read",
     "spire_status_string",
 )
 
@@ -119,6 +120,8 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_get_cta_times.restype = ctypes.c_int
     lib.spire_get_cta_times.argtypes = [P, SZ, ctypes.POINTER(ctypes.c_uint64), I32,
                                         ctypes.POINTER(I32), P]
+    lib.spire_stream_read.restype = ctypes.c_int
+    lib.spire_stream_read.argtypes = [P, SZ, P]
     lib.spire_status_string.restype = ctypes.c_char_p
     lib.spire_status_string.argtypes = [ctypes.c_int]
     return lib
@@ -252,6 +255,12 @@ def spire_get_cta_times(workspace, ws_bytes, max_ctas=1024, stream=None):
         raise SpireError(st, "spire_get_cta_times")
     m = min(n.value, max_ctas)
     return [(int(buf[2 * i]), int(buf[2 * i + 1])) for i in range(m)]
+
+
+def spire_stream_read(src, nbytes, stream=None) -> int:
+    """One launch that only reads nbytes at src (the floor of a call that
+    moves that many bytes); see include/spire.h."""
+    return int(LIB.spire_stream_read(_ptr(src), int(nbytes), _stream(stream, src)))
 
 
 def status_string(status: int) -> str:

@@ -31,7 +31,8 @@ def test_header_declares_the_boundary():
         "spire_feedback_append_workspace_bytes", "spire_feedback_append",
         "spire_verify_tokens_workspace_bytes", "spire_verify_tokens",
         "spire_magicdec_workspace_bytes", "spire_magicdec_attention",
-        "spire_get_device_error", "spire_get_cta_times", "spire_status_string"]), names
+        "spire_get_device_error", "spire_get_cta_times", "spire_stream_read",
+        "spire_status_string"]), names
 
 
 def test_library_exports_every_declared_symbol(spire):
@@ -252,3 +253,12 @@ def test_cta_times_host_checks(spire):
     assert lib.spire_get_cta_times(256, 1 << 20, buf, -1, ctypes.byref(n), None) == 1
     assert lib.spire_get_cta_times(256, 255, buf, 2, ctypes.byref(n), None) == 3
     assert n.value == -1
+
+
+def test_stream_read_host_checks(spire):
+    # a zero-byte read is a no-op; null, misaligned or ragged sizes are refused
+    # before anything is launched
+    assert spire.spire_stream_read(None, 0, 0) == 0
+    assert spire.spire_stream_read(None, 16, 0) == 1
+    assert spire.spire_stream_read(1 << 20, 8, 0) == 1
+    assert spire.spire_stream_read((1 << 20) + 8, 16, 0) == 1
