@@ -304,7 +304,9 @@ __global__ void __launch_bounds__(224, 1)
                 if (!mbar_wait(bar_sfull + 8 * sb, (n_qk >> 1) & 1)) { ok = false; break; }
                 tc_fence_after();
                 float sv[KW];
-                if (active) {
+                // this thread's slice of the S row, with keys past the row's causal /
+                // length limit masked
+                auto load_scores = [&]() {
                     if constexpr (KW == 16) {
                         tmem_ld16(trow + C::S_COL + sb * 64 + kofs, sv);
                     } else {
@@ -317,40 +319,14 @@ __global__ void __launch_bounds__(224, 1)
                         }
                     }
                     tmem_wait_ld();
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar_sfree + 8 * sb);
-                ++n_qk;
-                float factor = 1.f;
-                if (active) {
                     if (key0 + KW > lim) {
 #pragma unroll
                         for (int j = 0; j < KW; ++j)
                             if (key0 + j >= lim) sv[j] = NEG_INF;
                     }
-                    // independent partial maxima (three-input max) keep the chain short
-                    constexpr int NP = KW / 8;        // partials of 8 scores each
-                    float mp[NP];
-#pragma unroll
-                    for (int j = 0; j < NP; ++j) {
-                        const float* v = sv + 8 * j;
-                        mp[j] = fmaxf(fmax3(fmax3(v[0], v[1], v[2]), v[3], v[4]),
-                                      fmax3(v[5], v[6], v[7]));
-                    }
-#pragma unroll
-                    for (int w = NP / 2; w > 0; w /= 2)
-#pragma unroll
-                        for (int j = 0; j < w; ++j) mp[j] = fmaxf(mp[j], mp[j + w]);
-                    const float mx = mp[0];
-                    const float t = mx * sl2;
-                    if (t > m + kLazy) {                  // also true while m is -inf
-                        factor = ex2(m - t);              // 0 when m is -inf
-                        l *= factor;
-                        m = t;
-                    }
-                    const float mr = (m == NEG_INF) ? 0.f : m;
-                    // exponent arguments and partial sums two lanes at a time
+                };
+                // exponentials 2^(s sl2 - mr) in place and their sum, two lanes at a time
+                auto exponentials = [&](float mr) -> float {
                     const uint64_t scale2 = f2_pack(sl2, sl2), shift2 = f2_pack(-mr, -mr);
                     uint64_t sp[4];
 #pragma unroll
@@ -363,12 +339,70 @@ __global__ void __launch_bounds__(224, 1)
                         sv[2 * j + 1] = ex2(y);
                         sp[j & 3] = add2(sp[j & 3], f2_pack(sv[2 * j], sv[2 * j + 1]));
                     }
-                    {
-                        float x, y;
-                        f2_unpack(add2(add2(sp[0], sp[1]), add2(sp[2], sp[3])), x, y);
-                        l += x + y;
-                    }
+                    float x, y;
+                    f2_unpack(add2(add2(sp[0], sp[1]), add2(sp[2], sp[3])), x, y);
+                    return x + y;
+                };
+                // With one copy (64 keys a thread) the row maximum is a tenth of
+                // the per-tile work, so it is skipped where it cannot matter (fast
+                // path below) and the S buffer is released only after the
+                // exponentials, so that a warp can reload its scores.  With more
+                // copies (16 or 32 keys a thread) the maximum is cheap and the
+                // buffer is released at once, so the QK two tiles ahead never waits.
+                constexpr bool kFast = (KW == 64);
+                if (active) load_scores();
+                if (!kFast) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar_sfree + 8 * sb);   // S buffer read
                 }
+                float factor = 1.f;
+                if (active) {
+                    // Fast path: exponentials against the running max m as it
+                    // stands.  The max only moves when a score exceeds m by more
+                    // than 2^8 (lazy rescaling), which makes some exponential
+                    // > 2^8; a sum <= 2^8 rules that out, so m stays and these
+                    // are exactly the values the max-first path below computes.
+                    // Otherwise (the first tile of a segment, a sum above 2^8,
+                    // NaN) the warp takes that path, after reloading its scores
+                    // (tensor-memory loads are warp-wide).
+                    float sum = 0.f;
+                    bool slow = !kFast || (m == NEG_INF);
+                    if (!slow) {
+                        sum = exponentials(m);
+                        slow = !(sum <= 256.f);           // 2^kLazy
+                    }
+                    if (!kFast || __any_sync(0xffffffffu, slow)) {
+                        if (kFast && __any_sync(0xffffffffu, m != NEG_INF)) load_scores();
+                        // independent partial maxima (three-input max) keep the chain short
+                        constexpr int NP = KW / 8;        // partials of 8 scores each
+                        float mp[NP];
+#pragma unroll
+                        for (int j = 0; j < NP; ++j) {
+                            const float* v = sv + 8 * j;
+                            mp[j] = fmaxf(fmax3(fmax3(v[0], v[1], v[2]), v[3], v[4]),
+                                          fmax3(v[5], v[6], v[7]));
+                        }
+#pragma unroll
+                        for (int w = NP / 2; w > 0; w /= 2)
+#pragma unroll
+                            for (int j = 0; j < w; ++j) mp[j] = fmaxf(mp[j], mp[j + w]);
+                        const float t = mp[0] * sl2;
+                        if (t > m + kLazy) {              // also true while m is -inf
+                            factor = ex2(m - t);          // 0 when m is -inf
+                            l *= factor;
+                            m = t;
+                        }
+                        sum = exponentials((m == NEG_INF) ? 0.f : m);
+                    }
+                    l += sum;
+                }
+                if (kFast) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar_sfree + 8 * sb);   // S buffer read
+                }
+                ++n_qk;
                 const uint32_t pb = n_pv & 1;
                 if (active) {
                     // PV two tiles back read this P buffer: it must have completed
