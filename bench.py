@@ -264,7 +264,12 @@ def verify_config_entry(spire, name, dev, stream, flush, args, hbm_peak, max_seq
     if spire.spire_get_device_error(ws, stream):
         raise RuntimeError("device error word set by the %s verify call" % name)
     n = max(1, min(args.steps, 100))
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    sampler.start()
+    time.sleep(0.3)
+    t0 = time.time()
     ms = reduce_max([event_ms(call, n, flush, stream)], dist, dev)[0]   # the slowest rank
+    clocks = sampler.stop(t0, time.time())
     flush(7)
     call()
     bal = cta_balance(spire.spire_get_cta_times(ws, ws.numel()))
@@ -278,7 +283,7 @@ def verify_config_entry(spire, name, dev, stream, flush, args, hbm_peak, max_seq
              "tflops": verify_flops(L, k, Hq, D) / (ms * 1e-3) / 1e12,
              "rows_per_kv_head": (Hq // Hkv) * (k + 1),
              "load_balance": bal,
-             "traffic": dram_traffic("verify:%s" % name)}
+             "traffic": dram_traffic("verify:%s" % name), "clocks": clocks}
     del vi, ws, out
     torch.cuda.empty_cache()
     return entry
