@@ -379,6 +379,23 @@ SPIRE_API spire_status spire_verify_tokens(const float *p, const float *q,
                                            size_t ws_bytes, void *stream);
 
 /*
+ * spire_test_stall_next_call -- a test hook for the failure path; the paper
+ * has no counterpart, and production code does not call it.  In the next
+ * spire_verify_attention or spire_draft_sparse_attention call made by the
+ * calling host thread, the producer of every CTA that reaches pair `pair`
+ * (= b * num_kv_heads + g) issues no loads from that pair on, so no copy of
+ * it is ever in flight and the bounded waits for it run out (2 s).  The call
+ * returns normally; its kernels give up, record SPIRE_DEVERR_TIMEOUT in the
+ * device error word (spire_get_device_error), leave the affected outputs
+ * unspecified, drain their own copies and tensor-core work, free tensor
+ * memory, and leave the context usable.  The stalling kernels are separate
+ * test instantiations (head_dim 128 only; at other head dims the call runs
+ * normally), so the production kernels carry no trace of the hook.  Returns
+ * SPIRE_ERR_INVALID_ARG for pair < 0 (nothing is armed then).
+ */
+SPIRE_API spire_status spire_test_stall_next_call(int32_t pair);
+
+/*
  * spire_stream_read -- a measurement helper; the paper has no counterpart.
  * One kernel launch that reads `bytes` of device memory at `src` once and
  * computes nothing: one CTA per SM streams a contiguous run of 16 KB chunks

@@ -45,6 +45,7 @@ EXPORTED = (
     "spire_get_device_error",
     "spire_get_cta_times",
     "spire_stream_read",
+    "spire_test_stall_next_call",
     "spire_status_string",
 )
 
@@ -122,6 +123,8 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
                                         ctypes.POINTER(I32), P]
     lib.spire_stream_read.restype = ctypes.c_int
     lib.spire_stream_read.argtypes = [P, SZ, P]
+    lib.spire_test_stall_next_call.restype = ctypes.c_int
+    lib.spire_test_stall_next_call.argtypes = [I32]
     lib.spire_status_string.restype = ctypes.c_char_p
     lib.spire_status_string.argtypes = [ctypes.c_int]
     return lib
@@ -261,6 +264,12 @@ def spire_stream_read(src, nbytes, stream=None) -> int:
     """One launch that only reads nbytes at src (the floor of a call that
     moves that many bytes); see include/spire.h."""
     return int(LIB.spire_stream_read(_ptr(src), int(nbytes), _stream(stream, src)))
+
+
+def spire_test_stall_next_call(pair) -> int:
+    """Test hook: the next attention call on this thread stalls `pair` (its
+    waits run out); see include/spire.h."""
+    return int(LIB.spire_test_stall_next_call(int(pair)))
 
 
 def status_string(status: int) -> str:

@@ -720,6 +720,14 @@ MdLayout md_layout(const spire_attn_desc* d, int S) {
     return l;
 }
 
+// Test hook (spire_test_stall_next_call): the next attention call made by this
+// host thread stalls one pair.
+struct TestStall {
+    bool armed = false;
+    int32_t pair = -1;
+};
+thread_local TestStall g_test_stall;
+
 // Launches the attention for one call: a one-CTA kernel zeroing the pair
 // counters, then the attention kernel, each a programmatic dependent of the
 // kernel before it (each waits for that kernel to complete before it touches
@@ -783,6 +791,13 @@ spire_status run(int mode, const void* q, const CUtensorMap& tk, const CUtensorM
     ap.head = use_tc ? kHeadTc : kHeadMma;
     cudaError_t e;
     const int nc = R <= 32 ? 4 : (R <= 64 ? 2 : 1);   // query copies of the tcgen05 kernel
+    if (g_test_stall.armed) {      // spire_test_stall_next_call: this thread's next call only
+        g_test_stall.armed = false;
+        if (D == 128) {
+            e = launch_stall_d128(use_tc, nc, g_test_stall.pair, tk, tv, tq, ap, ctas, stream);
+            return e == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
+        }
+    }
     if (use_tc)
         e = D == 128 ? launch_attn_tc_d128(nc, tk, tv, tq, ap, ctas, stream)
                      : launch_attn_tc_d64(nc, tk, tv, tq, ap, ctas, stream);
@@ -1022,6 +1037,13 @@ spire_status spire_get_cta_times(const void* workspace, size_t ws_bytes, uint64_
                   cudaStreamSynchronize(s) != cudaSuccess))
         return SPIRE_ERR_CUDA;
     *n_out = n;
+    return SPIRE_OK;
+}
+
+spire_status spire_test_stall_next_call(int32_t pair) {
+    if (pair < 0) return SPIRE_ERR_INVALID_ARG;
+    g_test_stall.armed = true;
+    g_test_stall.pair = pair;
     return SPIRE_OK;
 }
 

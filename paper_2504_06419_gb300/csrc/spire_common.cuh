@@ -313,6 +313,11 @@ struct ProducerSmem {
     bool tail_first;       // walk a range's split last pair first (TileWalker)
 };
 
+// Pair whose loads the test instantiations (kStall) never issue, set by the
+// host before such a launch (spire_test_stall_next_call); one copy per
+// translation unit.  The production instantiations never read it.
+static __device__ int32_t g_stall_pair = -1;
+
 // Meta word layout: meta[2s] = {b, g, key0, leff}; meta[2s+1] = {flags |
 // (qflag << 8), slot, nseg, first_slot} where qflag = 16 | Q buffer when the
 // tile starts a segment whose query rows were loaded.
@@ -321,8 +326,10 @@ struct ProducerSmem {
 // found.  The stage ring protocol: wait `empty` (parity ph ^ 1), fill, arrive
 // on `full` with the byte count; a tile that must not be read (bad length or
 // page) arrives without a copy and carries kBad.  The run ends with a stage
-// that carries kTerm.
-template <int D, int NST>
+// that carries kTerm.  With kStall (test instantiations only) the producer
+// stops before the first tile of pair g_stall_pair, issuing nothing more, so
+// the consumers' waits for that tile run out.
+template <int D, int NST, bool kStall = false>
 __device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CUtensorMap* tmap_k,
                             const CUtensorMap* tmap_v, const CUtensorMap* tmap_q,
                             const ProducerSmem& sm) {
@@ -344,6 +351,12 @@ __device__ uint32_t produce(const AttnParams& p, const SchedShared& sh, const CU
         if (!mbar_wait(sm.bar_empty + 8 * st, ph ^ 1)) { ok = false; break; }
         TileMeta m;
         const int t = wk.next(p, &m);
+        if constexpr (kStall) {
+            if (m.b * p.Hkv + m.g == g_stall_pair) {
+                ok = false;
+                break;
+            }
+        }
         int qflag = 0;
         if ((m.flags & kFirst) && !(m.flags & kBad)) {
             // the pair's query rows r = i*G + hl, one box per 64 columns

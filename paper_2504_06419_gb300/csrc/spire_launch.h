@@ -29,6 +29,13 @@ cudaError_t launch_attn_tc_d128(int nc, const CUtensorMap& tk, const CUtensorMap
                                 const CUtensorMap& tq, const AttnParams& p, int ctas,
                                 cudaStream_t stream);
 
+// Test instantiations at head_dim 128 (spire_test_stall_next_call): the
+// warp-MMA kernel (tc = false) or the tcgen05 kernel with nc copies, whose
+// producer issues nothing from pair `pair` on.
+cudaError_t launch_stall_d128(bool tc, int nc, int32_t pair, const CUtensorMap& tk,
+                              const CUtensorMap& tv, const CUtensorMap& tq, const AttnParams& p,
+                              int ctas, cudaStream_t stream);
+
 // Largest dynamic shared memory one block of this build may use (227 KB).
 constexpr int kMaxDynSmem = 232448;
 

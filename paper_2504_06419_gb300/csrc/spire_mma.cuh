@@ -60,7 +60,7 @@ struct MmaCfg {
                   "swizzled regions must be 1024-byte aligned");
 };
 
-template <int D, int MT, int KP, int NST>
+template <int D, int MT, int KP, int NST, bool kStall = false>
 __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     attn_mma_kernel(const __grid_constant__ CUtensorMap tmap_k,
                     const __grid_constant__ CUtensorMap tmap_v,
@@ -118,7 +118,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         if (lane != 0) return;
         const ProducerSmem psm{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
                                bar_empty, bar_qfull, bar_qempty, 1, 0, 2, true};
-        const uint32_t err = produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, psm);
+        const uint32_t err = produce<D, NST, kStall>(p, *sh, &tmap_k, &tmap_v, &tmap_q, psm);
         if (err) atomicOr(&p.err[blockIdx.x], (int)err);
         return;
     }

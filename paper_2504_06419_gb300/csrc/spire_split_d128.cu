@@ -12,4 +12,9 @@ cudaError_t launch_attn_tc_d128(int nc, const CUtensorMap& tk, const CUtensorMap
                                cudaStream_t stream) {
     return launch_tc_dispatch<128>(nc, tk, tv, tq, p, ctas, stream);
 }
+cudaError_t launch_stall_d128(bool tc, int nc, int32_t pair, const CUtensorMap& tk,
+                              const CUtensorMap& tv, const CUtensorMap& tq, const AttnParams& p,
+                              int ctas, cudaStream_t stream) {
+    return launch_stall_dispatch<128>(tc, nc, pair, tk, tv, tq, p, ctas, stream);
+}
 }  // namespace spire

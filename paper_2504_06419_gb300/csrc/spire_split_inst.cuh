@@ -28,7 +28,7 @@ cudaError_t launch_pdl(Kern kern, int ctas, int threads, int smem, cudaStream_t 
     return cudaLaunchKernelEx(&cfg, kern, tk, tv, tq, p);
 }
 
-template <int D, int MT>
+template <int D, int MT, bool kStall = false>
 cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
                           const AttnParams& p, int ctas, cudaStream_t stream) {
     constexpr int KP = key_parts(MT);
@@ -36,7 +36,7 @@ cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CU
     static_assert(NST >= 2, "stage ring does not fit in shared memory");
     using C = MmaCfg<D, MT, KP, NST>;
     static_assert(C::SMEM <= kMaxDynSmem, "shared memory budget exceeded");
-    auto kern = attn_mma_kernel<D, MT, KP, NST>;
+    auto kern = attn_mma_kernel<D, MT, KP, NST, kStall>;
     // the shared-memory opt-in is per device; remember it for the first 64
     static std::atomic<unsigned long long> done{0ull};
     int dev = 0;
@@ -52,14 +52,14 @@ cudaError_t launch_attn_t(const CUtensorMap& tk, const CUtensorMap& tv, const CU
     return launch_pdl(kern, ctas, C::THREADS, C::SMEM, stream, tk, tv, tq, p);
 }
 
-template <int D, int NC>
+template <int D, int NC, bool kStall = false>
 cudaError_t launch_tc_t(const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& tq,
                         const AttnParams& p, int ctas, cudaStream_t stream) {
     constexpr int NST = tc_stages<D, NC>();
     static_assert(NST >= 2, "stage ring does not fit in shared memory");
     using C = TcCfg<D, NC, NST>;
     static_assert(C::SMEM <= kMaxDynSmem, "shared memory budget exceeded");
-    auto kern = attn_tc_kernel<D, NC, NST>;
+    auto kern = attn_tc_kernel<D, NC, NST, kStall>;
     static std::atomic<unsigned long long> done{0ull};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -81,6 +81,24 @@ cudaError_t launch_tc_dispatch(int nc, const CUtensorMap& tk, const CUtensorMap&
         case 4: return launch_tc_t<D, 4>(tk, tv, tq, p, ctas, stream);
         case 2: return launch_tc_t<D, 2>(tk, tv, tq, p, ctas, stream);
         case 1: return launch_tc_t<D, 1>(tk, tv, tq, p, ctas, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+// Test instantiations (spire_test_stall_next_call): the same kernels with
+// kStall, after the host has set this unit's g_stall_pair.
+template <int D>
+cudaError_t launch_stall_dispatch(bool tc, int nc, int32_t pair, const CUtensorMap& tk,
+                                  const CUtensorMap& tv, const CUtensorMap& tq,
+                                  const AttnParams& p, int ctas, cudaStream_t stream) {
+    cudaError_t e = cudaMemcpyToSymbolAsync(g_stall_pair, &pair, sizeof(pair), 0,
+                                            cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return e;
+    if (!tc) return launch_attn_t<D, 1, true>(tk, tv, tq, p, ctas, stream);
+    switch (nc) {
+        case 4: return launch_tc_t<D, 4, true>(tk, tv, tq, p, ctas, stream);
+        case 2: return launch_tc_t<D, 2, true>(tk, tv, tq, p, ctas, stream);
+        case 1: return launch_tc_t<D, 1, true>(tk, tv, tq, p, ctas, stream);
         default: return cudaErrorInvalidValue;
     }
 }

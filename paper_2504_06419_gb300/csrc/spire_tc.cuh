@@ -78,7 +78,7 @@ struct TcCfg {
 
 constexpr float kLazy = 8.0f;   // log2 units: rescale O only when the max grows by > 2^8
 
-template <int D, int NC, int NST>
+template <int D, int NC, int NST, bool kStall = false>
 __global__ void __launch_bounds__(224, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v,
@@ -150,7 +150,7 @@ __global__ void __launch_bounds__(224, 1)
         if (lane == 0) {
             const ProducerSmem ps{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
                                   bar_empty, bar_qfull, bar_qempty, NC, 128 / NC, 1, false};
-            err |= produce<D, NST>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
+            err |= produce<D, NST, kStall>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------ QK issuer
