@@ -6,11 +6,12 @@
 //                       through the block table, and streams each K and V
 //                       tile with TMA (64 keys x D, 128-byte swizzle) into
 //                       an NST-deep ring of shared-memory stages.
-//   warps 0..NW-1       consumer warp w owns m-tile w / KP (16 query rows)
-//                       and key slice w % KP (64 / KP keys of every tile).
-//                       It keeps Q in registers for the current pair, runs
-//                       S = Q K^T and O += P V on the tensor cores and an
-//                       fp32 online softmax in base 2.
+//   warps 0..NW-1       consumer warp w owns key slice w (64 / KP = 16 keys
+//                       of every tile).  It keeps Q^T in registers for the
+//                       current pair, runs S^T = K Q^T and O^T += V^T P^T on
+//                       the tensor cores (keys and head dimensions as the
+//                       MMA's 16 rows, the pair's query rows as its 8
+//                       columns) and an fp32 online softmax in base 2.
 //   warp NW+1 (epilogue) at the end of a pair's segment the consumers only
 //                       hand their (O, m, l) rows to one of two shared-memory
 //                       buffers and go on with the next segment; this warp
@@ -18,8 +19,8 @@
 //                       output, or to a partial slot that the last-arriving
 //                       CTA merges (see spire_common.cuh), publishing with a
 //                       fence and an atomic, off the consumers' path.
-// The kernel serves pairs of at most 8 query rows (one m-tile, rows 8..15 of
-// the MMA are padding), so a buffer holds 8 rows per consumer warp.
+// The kernel serves pairs of at most 8 query rows (the MMA's N = 8), so a
+// buffer holds 8 rows per consumer warp.
 //
 // Precision: P enters the PV product as P_hi + P_lo, two bf16 terms carrying
 // ~16 mantissa bits, so rounding P to bf16 (~1.7e-3 rms relative) never
@@ -35,8 +36,6 @@ struct MmaCfg {
     static constexpr int NW = MT * KP;            // consumer warps
     static constexpr int THREADS = 32 * (NW + 2); // + a producer and an epilogue warp
     static constexpr int KW = kPage / KP;         // keys per consumer warp per tile
-    static constexpr int NT = KW / 8;             // S n-tiles per warp
-    static constexpr int KK = KW / 16;            // PV k-steps per warp
     static constexpr int TILE = kPage * D * 2;    // bytes of one K (or V) tile
     static constexpr int STAGE = 2 * TILE;
     static constexpr int SCR = D + 8;             // floats per scratch row
@@ -52,7 +51,7 @@ struct MmaCfg {
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
     static constexpr int OFF_BAR = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16 + 16;
     static constexpr int SMEM = OFF_BAR + (2 * NST + 9) * 8 + 1024;  // + alignment slack
-    static_assert(KW >= 16 && NT % 2 == 0, "each warp needs >= 16 keys of a tile");
+    static_assert(KW == 16, "each consumer warp owns one 16-key MMA slice of a tile");
     static_assert(MT == 1, "one m-tile: the kernel serves at most 8 query rows");
     static_assert(D % 64 == 0, "head_dim must be a multiple of 64");
     // 128-byte swizzled TMA destinations must sit on 1024-byte boundaries
@@ -204,36 +203,58 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     }
 
     // ---------------------------------------------------------- consumers
-    const int mt = warp / KP, kp = warp - (warp / KP) * KP;
-    const int gq = lane >> 2, tq = lane & 3;          // mma group / thread-in-group
-    const int r0 = mt * 16 + gq, r1 = r0 + 8;         // the two rows this thread holds
-    const int wkey = kp * C::KW;                      // first key of this warp in a tile
+    // Warp w owns keys [w KW, (w + 1) KW) of every tile (KW = 16).  The keys
+    // are the MMA rows (M = 16) and the pair's R <= 8 query rows its columns
+    // (N = 8), so at most 8 - R columns and no row of an MMA are padding:
+    //   S^T  = K Q^T          A = the warp's K slice, B = Q^T (registers)
+    //   O^T += V^T (P^T)      A = the V slice read transposed, B = P^T moved
+    //                         into the B layout with movmatrix.trans
+    // Lane (gq, tq) = (lane / 4, lane % 4) holds S^T of slice keys gq and
+    // gq + 8 for query rows ra = 2 tq and rb = 2 tq + 1, and O^T of
+    // dimensions 16 j + gq and 16 j + gq + 8 (j < D / 16) of the same rows.
+    const int gq = lane >> 2, tq = lane & 3;
+    const int ra = 2 * tq, rb = ra + 1;
+    const int wkey = warp * C::KW;                    // first key of this warp in a tile
     const float sl2 = p.sl2;
     const float NEG_INF = __int_as_float(0xff800000);
     const float NANF = __int_as_float(0x7fc00000);
+    constexpr uint32_t FULL = 0xffffffffu;
 
-    float o[D / 8][4];
-    uint32_t qf[D / 16][4];
-    float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
+    float o[D / 16][4];
+    uint32_t qf[D / 16][2];
+    float ma = NEG_INF, mb = NEG_INF, la = 0.f, lb = 0.f;
     bool poison = false;
     int cur_b = 0, cur_g = 0, cur_slot = 0, cur_nseg = 1, cur_first = 0;
-    int lim0 = 0, lim1 = 0, leff = 0;
+    int lima = 0, limb = 0, leff = 0;
     uint32_t st = 0, ph = 0, n_seg = 0;               // stage ring / segments handed over
     uint32_t cq[2] = {0u, 0u};                        // parity of each Q buffer
 
     // hand the segment's (O, m, l) rows, or the end of the work, to the epilogue
-    // warp through buffer n_seg & 1 (rows r0 = gq < 8 only: rows 8..15 are padding)
-    auto hand_over = [&](bool term, float lt0) -> bool {
+    // warp through buffer n_seg & 1 (rows < R only; the others are padding)
+    auto hand_over = [&](bool term, float lta, float ltb) -> bool {
         const int sb = n_seg & 1;
         if (!mbar_wait(bar_sempty + 8 * sb, ((n_seg >> 1) & 1) ^ 1)) return false;
         if (!term) {
-            float* so = scr_o + sb * C::SCR_BUF + (warp * C::SR + gq) * C::SCR;
+            float* so = scr_o + sb * C::SCR_BUF + warp * C::SR * C::SCR;
+            if (ra < p.R) {
 #pragma unroll
-            for (int j = 0; j < D / 8; ++j)
-                *reinterpret_cast<float2*>(so + 8 * j + 2 * tq) = make_float2(o[j][0], o[j][1]);
-            if (tq == 0)
-                scr_ml[sb * C::NW * C::SR + warp * C::SR + gq] =
-                    make_float2(poison ? NANF : m0, lt0);
+                for (int j = 0; j < D / 16; ++j) {
+                    so[ra * C::SCR + 16 * j + gq] = o[j][0];
+                    so[ra * C::SCR + 16 * j + gq + 8] = o[j][2];
+                }
+            }
+            if (rb < p.R) {
+#pragma unroll
+                for (int j = 0; j < D / 16; ++j) {
+                    so[rb * C::SCR + 16 * j + gq] = o[j][1];
+                    so[rb * C::SCR + 16 * j + gq + 8] = o[j][3];
+                }
+            }
+            if (gq == 0) {
+                float2* ml = scr_ml + sb * C::NW * C::SR + warp * C::SR;
+                ml[ra] = make_float2(poison ? NANF : ma, lta);
+                ml[rb] = make_float2(poison ? NANF : mb, ltb);
+            }
         }
         if (warp == 0 && lane == 0) {
             scr_info[2 * sb] = make_int4(cur_b, cur_g, cur_slot, cur_nseg);
@@ -250,24 +271,25 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
             if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
             return;
         }
-        const int4 ma = meta[2 * st], mb = meta[2 * st + 1];
-        const int flags = mb.x & 0xff;
+        const int4 mta = meta[2 * st], mtb = meta[2 * st + 1];
+        const int flags = mtb.x & 0xff;
         if (flags & kTerm) {
-            if (!hand_over(true, 0.f) && lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
+            if (!hand_over(true, 0.f, 0.f) && lane == 0)
+                atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
             return;
         }
         if (flags & kFirst) {
-            const int flags_q = mb.x;
-            cur_b = ma.x; cur_g = ma.y; leff = ma.w;
-            cur_slot = mb.y; cur_nseg = mb.z; cur_first = mb.w;
+            const int flags_q = mtb.x;
+            cur_b = mta.x; cur_g = mta.y; leff = mta.w;
+            cur_slot = mtb.y; cur_nseg = mtb.z; cur_first = mtb.w;
             poison = false;
-            m0 = m1 = NEG_INF; l0 = l1 = 0.f;
+            ma = mb = NEG_INF; la = lb = 0.f;
 #pragma unroll
-            for (int j = 0; j < D / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+            for (int j = 0; j < D / 16; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
             // rows r = i*G + hl (block row i, head hl of the group)
-            const int i0 = min(r0 / p.G, p.kp1 - 1), i1 = min(r1 / p.G, p.kp1 - 1);
-            lim0 = leff - (p.kp1 - 1) + i0;
-            lim1 = leff - (p.kp1 - 1) + i1;
+            const int ia = min(ra / p.G, p.kp1 - 1), ib = min(rb / p.G, p.kp1 - 1);
+            lima = leff - (p.kp1 - 1) + ia;
+            limb = leff - (p.kp1 - 1) + ib;
             const int qflag = flags_q >> 8;
             if (qflag & 16) {
                 const int qb = qflag & 1;
@@ -276,14 +298,16 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
                     return;
                 }
                 cq[qb] ^= 1;
+                // B = Q^T: lane (gq, tq) takes row gq, columns 2 tq, 2 tq + 1 of
+                // the 8x8 blocks at 16-byte chunks 2 ks and 2 ks + 1
                 const uint32_t qbase = qsm + qb * C::QBUF;
-                const int qrow = mt * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
+                const int qrow = lane & 7;
 #pragma unroll
-                for (int ks = 0; ks < D / 16; ++ks) {
-                    const int chunk = 2 * ks + (lane >> 4);
-                    ldsm_x4(qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3],
+                for (int ks = 0; ks < D / 16; ks += 2) {
+                    const int chunk = 2 * ks + (lane >> 3);
+                    ldsm_x4(qf[ks][0], qf[ks][1], qf[ks + 1][0], qf[ks + 1][1],
                             qbase + (chunk >> 3) * C::QHALF + qrow * 128 +
-                                (((chunk & 7) ^ (lane & 7)) << 4));
+                                (((chunk & 7) ^ qrow) << 4));
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar_qempty + 8 * qb);
@@ -292,121 +316,94 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         if (flags & kBad) {
             poison = true;
         } else {
-            const int key0 = ma.z;                           // sequence index of tile key 0
+            const int key0 = mta.z;                          // sequence index of tile key 0
             const uint32_t kb = base + st * C::STAGE, vb = kb + C::TILE;
-            // ---- S = Q K^T over this warp's KW keys
-            float s[C::NT][4];
-#pragma unroll
-            for (int j = 0; j < C::NT; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+            // ---- S^T = K Q^T over this warp's 16 keys: two accumulation chains
+            float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+            const int krow = wkey + ((lane >> 3) & 1) * 8 + (lane & 7);
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
-#pragma unroll
-                for (int jp = 0; jp < C::NT / 2; ++jp) {
-                    const int key = wkey + jp * 16 + ((lane >> 4) << 3) + (lane & 7);
-                    const int chunk = 2 * ks + ((lane >> 3) & 1);
-                    const uint32_t addr = kb + (chunk >> 3) * 8192 + key * 128 +
-                                          (((chunk & 7) ^ (lane & 7)) << 4);
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(b0, b1, b2, b3, addr);
-                    mma_bf16(s[2 * jp], qf[ks], b0, b1);
-                    mma_bf16(s[2 * jp + 1], qf[ks], b2, b3);
-                }
+                const int chunk = 2 * ks + (lane >> 4);
+                uint32_t a[4];
+                ldsm_x4(a[0], a[1], a[2], a[3],
+                        kb + (chunk >> 3) * 8192 + krow * 128 + (((chunk & 7) ^ (lane & 7)) << 4));
+                if (ks & 1) mma_bf16(s1, a, qf[ks][0], qf[ks][1]);
+                else        mma_bf16(s0, a, qf[ks][0], qf[ks][1]);
             }
+            float s[4] = {s0[0] + s1[0], s0[1] + s1[1], s0[2] + s1[2], s0[3] + s1[3]};
             // ---- causal / length mask (only tiles reaching past row 0's limit)
             if (key0 + kPage > leff - (p.kp1 - 1)) {
+                const int kx = key0 + wkey + gq;
+                if (kx >= lima) s[0] = NEG_INF;
+                if (kx >= limb) s[1] = NEG_INF;
+                if (kx + 8 >= lima) s[2] = NEG_INF;
+                if (kx + 8 >= limb) s[3] = NEG_INF;
+            }
+            // ---- online softmax (base 2); a row's 16 keys sit in the 8 lanes of its tq
+            float xa = fmaxf(s[0], s[2]), xb = fmaxf(s[1], s[3]);
 #pragma unroll
-                for (int j = 0; j < C::NT; ++j) {
-                    const int kidx = key0 + wkey + 8 * j + 2 * tq;
-                    if (kidx >= lim0) s[j][0] = NEG_INF;
-                    if (kidx + 1 >= lim0) s[j][1] = NEG_INF;
-                    if (kidx >= lim1) s[j][2] = NEG_INF;
-                    if (kidx + 1 >= lim1) s[j][3] = NEG_INF;
+            for (int off = 4; off < 32; off <<= 1) {
+                xa = fmaxf(xa, __shfl_xor_sync(FULL, xa, off));
+                xb = fmaxf(xb, __shfl_xor_sync(FULL, xb, off));
+            }
+            const float mna = fmaxf(ma, xa * sl2), mnb = fmaxf(mb, xb * sl2);
+            const float mra = (mna == NEG_INF) ? 0.f : mna;
+            const float mrb = (mnb == NEG_INF) ? 0.f : mnb;
+            const float aa = ex2(ma - mra), ab = ex2(mb - mrb);
+            ma = mna; mb = mnb;
+            s[0] = ex2(fmaf(s[0], sl2, -mra));
+            s[1] = ex2(fmaf(s[1], sl2, -mrb));
+            s[2] = ex2(fmaf(s[2], sl2, -mra));
+            s[3] = ex2(fmaf(s[3], sl2, -mrb));
+            la = la * aa + (s[0] + s[2]);
+            lb = lb * ab + (s[1] + s[3]);
+            if (__any_sync(FULL, (aa != 1.f) || (ab != 1.f))) {
+#pragma unroll
+                for (int j = 0; j < D / 16; ++j) {
+                    o[j][0] *= aa; o[j][1] *= ab;
+                    o[j][2] *= aa; o[j][3] *= ab;
                 }
             }
-            // ---- online softmax (base 2)
-            float mx0 = NEG_INF, mx1 = NEG_INF;
-#pragma unroll
-            for (int j = 0; j < C::NT; ++j) {
-                mx0 = fmaxf(mx0, fmaxf(s[j][0], s[j][1]));
-                mx1 = fmaxf(mx1, fmaxf(s[j][2], s[j][3]));
+            // ---- P^T = P_hi + P_lo (two bf16 terms) in the B layout
+            const uint32_t h0 = pack_bf16(s[0], s[1]);      // key gq: rows ra, rb
+            const uint32_t h1 = pack_bf16(s[2], s[3]);      // key gq + 8
+            const uint32_t l0 = pack_bf16(s[0] - bf16lo_to_f32(h0), s[1] - bf16hi_to_f32(h0));
+            const uint32_t l1 = pack_bf16(s[2] - bf16lo_to_f32(h1), s[3] - bf16hi_to_f32(h1));
+            const uint32_t bh0 = movm_trans(h0), bh1 = movm_trans(h1);
+            const uint32_t bl0 = movm_trans(l0), bl1 = movm_trans(l1);
+            // ---- O^T += V^T P^T; V of keys no row may see is zeroed (their
+            // slots may hold anything)
+            uint32_t mkA = 0xffffffffu, mkB = 0xffffffffu;
+            if (key0 + kPage > leff) {
+                const int kA = key0 + wkey + 2 * tq;        // keys of a0 / a1 (a2 / a3: + 8)
+                mkA = (kA < leff ? 0x0000ffffu : 0u) | (kA + 1 < leff ? 0xffff0000u : 0u);
+                mkB = (kA + 8 < leff ? 0x0000ffffu : 0u) | (kA + 9 < leff ? 0xffff0000u : 0u);
             }
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-            const float mn0 = fmaxf(m0, mx0 * sl2), mn1 = fmaxf(m1, mx1 * sl2);
-            const float mr0 = (mn0 == NEG_INF) ? 0.f : mn0;
-            const float mr1 = (mn1 == NEG_INF) ? 0.f : mn1;
-            const float a0 = ex2(m0 - mr0), a1 = ex2(m1 - mr1);
-            m0 = mn0; m1 = mn1;
-            float rs0 = 0.f, rs1 = 0.f;
+            const int vrow = wkey + ((lane >> 4) << 3) + (lane & 7);
 #pragma unroll
-            for (int j = 0; j < C::NT; ++j) {
-                s[j][0] = ex2(fmaf(s[j][0], sl2, -mr0));
-                s[j][1] = ex2(fmaf(s[j][1], sl2, -mr0));
-                s[j][2] = ex2(fmaf(s[j][2], sl2, -mr1));
-                s[j][3] = ex2(fmaf(s[j][3], sl2, -mr1));
-                rs0 += s[j][0] + s[j][1];
-                rs1 += s[j][2] + s[j][3];
-            }
-            l0 = l0 * a0 + rs0;
-            l1 = l1 * a1 + rs1;
-            if (__any_sync(0xffffffffu, (a0 != 1.f) || (a1 != 1.f))) {
-#pragma unroll
-                for (int j = 0; j < D / 8; ++j) {
-                    o[j][0] *= a0; o[j][1] *= a0;
-                    o[j][2] *= a1; o[j][3] *= a1;
-                }
-            }
-            // ---- O += P V with P = P_hi + P_lo (two bf16 products)
-            const bool vmask = key0 + kPage > leff;
-#pragma unroll
-            for (int kk = 0; kk < C::KK; ++kk) {
-                uint32_t A_hi[4], A_lo[4];
-                // A fragment order: a0 (row g, k 0-7), a1 (row g+8, k 0-7),
-                // a2 (row g, k 8-15), a3 (row g+8, k 8-15)
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const float* sj = s[2 * kk + h];
-                    const uint32_t x0 = pack_bf16(sj[0], sj[1]);
-                    const uint32_t x1 = pack_bf16(sj[2], sj[3]);
-                    A_hi[2 * h + 0] = x0;
-                    A_hi[2 * h + 1] = x1;
-                    A_lo[2 * h + 0] = pack_bf16(sj[0] - bf16lo_to_f32(x0), sj[1] - bf16hi_to_f32(x0));
-                    A_lo[2 * h + 1] = pack_bf16(sj[2] - bf16lo_to_f32(x1), sj[3] - bf16hi_to_f32(x1));
-                }
-                const int kA = key0 + wkey + 16 * kk + 2 * tq;   // keys of b0/b2 (b1/b3: +8)
-#pragma unroll
-                for (int nn = 0; nn < D / 16; ++nn) {
-                    const int key = wkey + 16 * kk + (((lane >> 3) & 1) << 3) + (lane & 7);
-                    const int chunk = 2 * nn + (lane >> 4);
-                    const uint32_t addr = vb + (chunk >> 3) * 8192 + key * 128 +
-                                          (((chunk & 7) ^ (lane & 7)) << 4);
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_trans(b0, b1, b2, b3, addr);
-                    if (vmask) {
-                        // zero V of keys no row may see (their slots may hold anything)
-                        const uint32_t mA = (kA < leff ? 0x0000ffffu : 0u) |
-                                            (kA + 1 < leff ? 0xffff0000u : 0u);
-                        const uint32_t mB = (kA + 8 < leff ? 0x0000ffffu : 0u) |
-                                            (kA + 9 < leff ? 0xffff0000u : 0u);
-                        b0 &= mA; b2 &= mA; b1 &= mB; b3 &= mB;
-                    }
-                    mma_bf16(o[2 * nn], A_hi, b0, b1);
-                    mma_bf16(o[2 * nn], A_lo, b0, b1);
-                    mma_bf16(o[2 * nn + 1], A_hi, b2, b3);
-                    mma_bf16(o[2 * nn + 1], A_lo, b2, b3);
-                }
+            for (int j = 0; j < D / 16; ++j) {
+                const int chunk = 2 * j + ((lane >> 3) & 1);
+                uint32_t a[4];
+                ldsm_x4_trans(a[0], a[1], a[2], a[3],
+                              vb + (chunk >> 3) * 8192 + vrow * 128 +
+                                  (((chunk & 7) ^ (lane & 7)) << 4));
+                a[0] &= mkA; a[1] &= mkA; a[2] &= mkB; a[3] &= mkB;
+                mma_bf16(o[j], a, bh0, bh1);
+                mma_bf16(o[j], a, bl0, bl1);
             }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_empty + 8 * st);
 
         if (flags & kLast) {
-            // ---- segment end: the row sums over the quad, then hand over
-            float lt0 = l0 + __shfl_xor_sync(0xffffffffu, l0, 1);
-            lt0 += __shfl_xor_sync(0xffffffffu, lt0, 2);
-            if (!hand_over(false, lt0)) {
+            // ---- segment end: each row's sum over its 8 lanes, then hand over
+            float lta = la, ltb = lb;
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                lta += __shfl_xor_sync(FULL, lta, off);
+                ltb += __shfl_xor_sync(FULL, ltb, off);
+            }
+            if (!hand_over(false, lta, ltb)) {
                 if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
                 return;
             }

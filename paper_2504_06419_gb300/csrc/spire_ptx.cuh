@@ -199,6 +199,15 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1, uint32
                  : "r"(addr));
 }
 
+// Transpose of an 8x8 b16 matrix held one 32-bit pair per lane (lane l holds
+// row l/4, columns 2(l%4) and 2(l%4)+1); returns the same lane's pair of the
+// transposed matrix.
+__device__ __forceinline__ uint32_t movm_trans(uint32_t a) {
+    uint32_t r;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(r) : "r"(a));
+    return r;
+}
+
 // D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
 __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
                                          uint32_t b1) {
