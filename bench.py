@@ -998,16 +998,17 @@ def profile_call(args, cfg):
                 return spire.spire_verify_attention(q, vi.k_cache, vi.v_cache, vi.block_table, ctx,
                                                     kk, desc, out, ws, ws.numel(), sptr)
     elif what == "draft":
-        di = wl.make_draft(wl.draft_ctx_for_step(L, k, 0), Hq, Hkv, D, cfg.n_sink, cfg.window,
+        window = args.window or cfg.window
+        di = wl.make_draft(wl.draft_ctx_for_step(L, k, 0), Hq, Hkv, D, cfg.n_sink, window,
                            seed=cfg.seed + 17, device=dev)
         desc = spire.draft_desc(di.q, di.kv)
-        ws = torch.empty(spire.spire_draft_workspace_bytes(desc, cfg.n_sink, cfg.window),
+        ws = torch.empty(spire.spire_draft_workspace_bytes(desc, cfg.n_sink, window),
                          dtype=torch.uint8, device=dev)
         out = torch.empty(di.q.shape, dtype=torch.float32, device=dev)
 
         def call():
             return spire.spire_draft_sparse_attention(di.q, di.kv, di.ctx_lens, cfg.n_sink,
-                                                      cfg.window, desc, out, ws, ws.numel(), sptr)
+                                                      window, desc, out, ws, ws.numel(), sptr)
     elif what == "append":
         n_dl, n_act, d_model = 2, 3, Hq * D
         ai = wl.make_append(wl.draft_ctx_for_step(L, k, 0), n_act, n_dl, d_model, Hkv, D,
@@ -1064,6 +1065,8 @@ def main():
                          "the L2 flush) and exit: small profiler captures, never a benchmark")
     ap.add_argument("--calls", type=int, default=2,
                     help="calls after the warm-up in --profile-call mode")
+    ap.add_argument("--window", type=int, default=0,
+                    help="draft window for --profile-call draft (default: the workload's)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -315,20 +315,33 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         }
         if (flags & kBad) {
             poison = true;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_empty + 8 * st);
         } else {
             const int key0 = mta.z;                          // sequence index of tile key 0
             const uint32_t kb = base + st * C::STAGE, vb = kb + C::TILE;
+            // ---- this warp's K and V fragments into registers, then the stage is
+            // released: it is refilled while the tile is computed, which keeps
+            // more bytes in flight than holding it through the math
+            uint32_t kf[D / 16][4], vf[D / 16][4];
+            const int krow = wkey + ((lane >> 3) & 1) * 8 + (lane & 7);
+            const int vrow = wkey + ((lane >> 4) << 3) + (lane & 7);
+#pragma unroll
+            for (int j = 0; j < D / 16; ++j) {
+                const int kc = 2 * j + (lane >> 4), vc = 2 * j + ((lane >> 3) & 1);
+                ldsm_x4(kf[j][0], kf[j][1], kf[j][2], kf[j][3],
+                        kb + (kc >> 3) * 8192 + krow * 128 + (((kc & 7) ^ (lane & 7)) << 4));
+                ldsm_x4_trans(vf[j][0], vf[j][1], vf[j][2], vf[j][3],
+                              vb + (vc >> 3) * 8192 + vrow * 128 + (((vc & 7) ^ (lane & 7)) << 4));
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_empty + 8 * st);
             // ---- S^T = K Q^T over this warp's 16 keys: two accumulation chains
             float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
-            const int krow = wkey + ((lane >> 3) & 1) * 8 + (lane & 7);
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
-                const int chunk = 2 * ks + (lane >> 4);
-                uint32_t a[4];
-                ldsm_x4(a[0], a[1], a[2], a[3],
-                        kb + (chunk >> 3) * 8192 + krow * 128 + (((chunk & 7) ^ (lane & 7)) << 4));
-                if (ks & 1) mma_bf16(s1, a, qf[ks][0], qf[ks][1]);
-                else        mma_bf16(s0, a, qf[ks][0], qf[ks][1]);
+                if (ks & 1) mma_bf16(s1, kf[ks], qf[ks][0], qf[ks][1]);
+                else        mma_bf16(s0, kf[ks], qf[ks][0], qf[ks][1]);
             }
             float s[4] = {s0[0] + s1[0], s0[1] + s1[1], s0[2] + s1[2], s0[3] + s1[3]};
             // ---- causal / length mask (only tiles reaching past row 0's limit)
@@ -373,27 +386,21 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
             const uint32_t bl0 = movm_trans(l0), bl1 = movm_trans(l1);
             // ---- O^T += V^T P^T; V of keys no row may see is zeroed (their
             // slots may hold anything)
-            uint32_t mkA = 0xffffffffu, mkB = 0xffffffffu;
             if (key0 + kPage > leff) {
                 const int kA = key0 + wkey + 2 * tq;        // keys of a0 / a1 (a2 / a3: + 8)
-                mkA = (kA < leff ? 0x0000ffffu : 0u) | (kA + 1 < leff ? 0xffff0000u : 0u);
-                mkB = (kA + 8 < leff ? 0x0000ffffu : 0u) | (kA + 9 < leff ? 0xffff0000u : 0u);
+                const uint32_t mkA = (kA < leff ? 0x0000ffffu : 0u) | (kA + 1 < leff ? 0xffff0000u : 0u);
+                const uint32_t mkB = (kA + 8 < leff ? 0x0000ffffu : 0u) | (kA + 9 < leff ? 0xffff0000u : 0u);
+#pragma unroll
+                for (int j = 0; j < D / 16; ++j) {
+                    vf[j][0] &= mkA; vf[j][1] &= mkA; vf[j][2] &= mkB; vf[j][3] &= mkB;
+                }
             }
-            const int vrow = wkey + ((lane >> 4) << 3) + (lane & 7);
 #pragma unroll
             for (int j = 0; j < D / 16; ++j) {
-                const int chunk = 2 * j + ((lane >> 3) & 1);
-                uint32_t a[4];
-                ldsm_x4_trans(a[0], a[1], a[2], a[3],
-                              vb + (chunk >> 3) * 8192 + vrow * 128 +
-                                  (((chunk & 7) ^ (lane & 7)) << 4));
-                a[0] &= mkA; a[1] &= mkA; a[2] &= mkB; a[3] &= mkB;
-                mma_bf16(o[j], a, bh0, bh1);
-                mma_bf16(o[j], a, bl0, bl1);
+                mma_bf16(o[j], vf[j], bh0, bh1);
+                mma_bf16(o[j], vf[j], bl0, bl1);
             }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar_empty + 8 * st);
 
         if (flags & kLast) {
             // ---- segment end: each row's sum over its 8 lanes, then hand over
