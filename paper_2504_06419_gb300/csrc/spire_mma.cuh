@@ -33,8 +33,10 @@ namespace spire {
 
 template <int D, int MT, int KP, int NST>
 struct MmaCfg {
-    static constexpr int NW = MT * KP;            // consumer warps
-    static constexpr int THREADS = 32 * (NW + 2); // + a producer and an epilogue warp
+    static constexpr int NW = MT * KP;            // consumer warps of a group (one per key slice)
+    static constexpr int NG = 2;                  // consumer groups: they take alternate segments
+    static constexpr int NCW = NW * NG;           // consumer warps
+    static constexpr int THREADS = 32 * (NCW + 2);  // + a producer and an epilogue warp
     static constexpr int KW = kPage / KP;         // keys per consumer warp per tile
     static constexpr int TILE = kPage * D * 2;    // bytes of one K (or V) tile
     static constexpr int STAGE = 2 * TILE;
@@ -86,7 +88,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < NST; ++s) {
             mbar_init(bar_full + 8 * s, 1);
-            mbar_init(bar_empty + 8 * s, C::NW);
+            mbar_init(bar_empty + 8 * s, C::NCW);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(bar_qfull + 8 * b, 1);
@@ -112,7 +114,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     sched_setup(p, sh);   // ends with __syncthreads()
     if (threadIdx.x == 0) p.stamps[2 * blockIdx.x] = globaltimer_ns();
 
-    if (warp == C::NW) {
+    if (warp == C::NCW) {
         // ------------------------------------------------------ producer
         if (lane != 0) return;
         const ProducerSmem psm{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
@@ -121,7 +123,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         if (err) atomicOr(&p.err[blockIdx.x], (int)err);
         return;
     }
-    if (warp == C::NW + 1) {
+    if (warp == C::NCW + 1) {
         // ------------------------------------------------------ epilogue
         const float NEG_INF = __int_as_float(0xff800000);
         const float NANF = __int_as_float(0x7fc00000);
@@ -203,7 +205,13 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     }
 
     // ---------------------------------------------------------- consumers
-    // Warp w owns keys [w KW, (w + 1) KW) of every tile (KW = 16).  The keys
+    // Two groups of NW warps take alternate segments (group n % 2 computes the
+    // n-th segment of the CTA's walk), so each SM sub-partition runs two
+    // independent consumer warps; every consumer warp still waits for every
+    // stage and reads its tile record, and the other group's warps release a
+    // stage as soon as they have read it.  Each group has its own hand-over
+    // buffer (n % 2) for the epilogue warp, which takes them in segment order.
+    // Warp w of a group owns keys [w KW, (w + 1) KW) of every tile (KW = 16).  The keys
     // are the MMA rows (M = 16) and the pair's R <= 8 query rows its columns
     // (N = 8), so at most 8 - R columns and no row of an MMA are padding:
     //   S^T  = K Q^T          A = the warp's K slice, B = Q^T (registers)
@@ -214,7 +222,8 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     // dimensions 16 j + gq and 16 j + gq + 8 (j < D / 16) of the same rows.
     const int gq = lane >> 2, tq = lane & 3;
     const int ra = 2 * tq, rb = ra + 1;
-    const int wkey = warp * C::KW;                    // first key of this warp in a tile
+    const int grp = warp / C::NW, slice = warp - grp * C::NW;
+    const int wkey = slice * C::KW;                   // first key of this warp in a tile
     const float sl2 = p.sl2;
     const float NEG_INF = __int_as_float(0xff800000);
     const float NANF = __int_as_float(0x7fc00000);
@@ -223,19 +232,20 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     float o[D / 16][4];
     uint32_t qf[D / 16][2];
     float ma = NEG_INF, mb = NEG_INF, la = 0.f, lb = 0.f;
-    bool poison = false;
+    bool poison = false, own = false;                 // own: this group computes the segment
     int cur_b = 0, cur_g = 0, cur_slot = 0, cur_nseg = 1, cur_first = 0;
     int lima = 0, limb = 0, leff = 0;
-    uint32_t st = 0, ph = 0, n_seg = 0;               // stage ring / segments handed over
+    uint32_t st = 0, ph = 0, n_seg = 0;               // stage ring / segments ended so far
     uint32_t cq[2] = {0u, 0u};                        // parity of each Q buffer
 
     // hand the segment's (O, m, l) rows, or the end of the work, to the epilogue
-    // warp through buffer n_seg & 1 (rows < R only; the others are padding)
+    // warp through buffer n_seg & 1, this group's (rows < R only; the others
+    // are padding)
     auto hand_over = [&](bool term, float lta, float ltb) -> bool {
         const int sb = n_seg & 1;
         if (!mbar_wait(bar_sempty + 8 * sb, ((n_seg >> 1) & 1) ^ 1)) return false;
         if (!term) {
-            float* so = scr_o + sb * C::SCR_BUF + warp * C::SR * C::SCR;
+            float* so = scr_o + sb * C::SCR_BUF + slice * C::SR * C::SCR;
             if (ra < p.R) {
 #pragma unroll
                 for (int j = 0; j < D / 16; ++j) {
@@ -251,18 +261,17 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
                 }
             }
             if (gq == 0) {
-                float2* ml = scr_ml + sb * C::NW * C::SR + warp * C::SR;
+                float2* ml = scr_ml + sb * C::NW * C::SR + slice * C::SR;
                 ml[ra] = make_float2(poison ? NANF : ma, lta);
                 ml[rb] = make_float2(poison ? NANF : mb, ltb);
             }
         }
-        if (warp == 0 && lane == 0) {
+        if (slice == 0 && lane == 0) {
             scr_info[2 * sb] = make_int4(cur_b, cur_g, cur_slot, cur_nseg);
             scr_info[2 * sb + 1] = make_int4(cur_first, term ? 1 : 0, 0, 0);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_sfull + 8 * sb);
-        ++n_seg;
         return true;
     };
 
@@ -274,11 +283,13 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         const int4 mta = meta[2 * st], mtb = meta[2 * st + 1];
         const int flags = mtb.x & 0xff;
         if (flags & kTerm) {
-            if (!hand_over(true, 0.f, 0.f) && lane == 0)
+            // the group that would take the next segment tells the epilogue
+            if ((int)(n_seg & 1) == grp && !hand_over(true, 0.f, 0.f) && lane == 0)
                 atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
             return;
         }
         if (flags & kFirst) {
+            own = (int)(n_seg & 1) == grp;
             const int flags_q = mtb.x;
             cur_b = mta.x; cur_g = mta.y; leff = mta.w;
             cur_slot = mtb.y; cur_nseg = mtb.z; cur_first = mtb.w;
@@ -291,7 +302,9 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
             lima = leff - (p.kp1 - 1) + ia;
             limb = leff - (p.kp1 - 1) + ib;
             const int qflag = flags_q >> 8;
-            if (qflag & 16) {
+            if ((qflag & 16) && !own) {
+                cq[qflag & 1] ^= 1;     // the other group reads this Q buffer phase
+            } else if (qflag & 16) {
                 const int qb = qflag & 1;
                 if (!mbar_wait(bar_qfull + 8 * qb, cq[qb])) {
                     if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
@@ -313,7 +326,10 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
                 if (lane == 0) mbar_arrive(bar_qempty + 8 * qb);
             }
         }
-        if (flags & kBad) {
+        if (!own) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_empty + 8 * st);
+        } else if (flags & kBad) {
             poison = true;
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_empty + 8 * st);
@@ -403,17 +419,20 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         }
 
         if (flags & kLast) {
-            // ---- segment end: each row's sum over its 8 lanes, then hand over
-            float lta = la, ltb = lb;
+            if (own) {
+                // ---- segment end: each row's sum over its 8 lanes, then hand over
+                float lta = la, ltb = lb;
 #pragma unroll
-            for (int off = 4; off < 32; off <<= 1) {
-                lta += __shfl_xor_sync(FULL, lta, off);
-                ltb += __shfl_xor_sync(FULL, ltb, off);
+                for (int off = 4; off < 32; off <<= 1) {
+                    lta += __shfl_xor_sync(FULL, lta, off);
+                    ltb += __shfl_xor_sync(FULL, ltb, off);
+                }
+                if (!hand_over(false, lta, ltb)) {
+                    if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
+                    return;
+                }
             }
-            if (!hand_over(false, lta, ltb)) {
-                if (lane == 0) atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
-                return;
-            }
+            ++n_seg;
         }
         if (++st == NST) { st = 0; ph ^= 1; }
     }
