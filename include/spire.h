@@ -349,7 +349,7 @@ SPIRE_API spire_status spire_magicdec_attention(const void *q, const void *k_cac
 
 /*
  * spire_verify_tokens_workspace_bytes -- workspace size for
- * spire_verify_tokens (one partial per sequence and 8192-entry vocabulary
+ * spire_verify_tokens (one partial per sequence and 4096-entry vocabulary
  * chunk, and the device error word).  Returns 0 for invalid shapes.
  */
 SPIRE_API size_t spire_verify_tokens_workspace_bytes(int32_t batch, int32_t k, int32_t vocab);

@@ -34,7 +34,7 @@ namespace spire {
 template <int D, int MT, int KP, int NST>
 struct MmaCfg {
     static constexpr int NW = MT * KP;            // consumer warps of a group (one per key slice)
-    static constexpr int NG = 2;                  // consumer groups: they take alternate segments
+    static constexpr int NG = 2;                  // consumer groups: they take turns by segment
     static constexpr int NCW = NW * NG;           // consumer warps
     static constexpr int THREADS = 32 * (NCW + 2);  // + a producer and an epilogue warp
     static constexpr int KW = kPage / KP;         // keys per consumer warp per tile
@@ -205,12 +205,12 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     }
 
     // ---------------------------------------------------------- consumers
-    // Two groups of NW warps take alternate segments (group n % 2 computes the
-    // n-th segment of the CTA's walk), so each SM sub-partition runs two
+    // NG groups of NW warps take turns by segment (group n % NG computes the
+    // n-th segment of the CTA's walk), so each SM sub-partition runs NG
     // independent consumer warps; every consumer warp still waits for every
-    // stage and reads its tile record, and the other group's warps release a
-    // stage as soon as they have read it.  Each group has its own hand-over
-    // buffer (n % 2) for the epilogue warp, which takes them in segment order.
+    // stage and reads its tile record, and the other groups' warps release a
+    // stage as soon as they have read it.  Segment n is handed to the epilogue
+    // warp through buffer n % 2; the epilogue takes them in segment order.
     // Warp w of a group owns keys [w KW, (w + 1) KW) of every tile (KW = 16).  The keys
     // are the MMA rows (M = 16) and the pair's R <= 8 query rows its columns
     // (N = 8), so at most 8 - R columns and no row of an MMA are padding:
@@ -239,8 +239,7 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
     uint32_t cq[2] = {0u, 0u};                        // parity of each Q buffer
 
     // hand the segment's (O, m, l) rows, or the end of the work, to the epilogue
-    // warp through buffer n_seg & 1, this group's (rows < R only; the others
-    // are padding)
+    // warp through buffer n_seg & 1 (rows < R only; the others are padding)
     auto hand_over = [&](bool term, float lta, float ltb) -> bool {
         const int sb = n_seg & 1;
         if (!mbar_wait(bar_sempty + 8 * sb, ((n_seg >> 1) & 1) ^ 1)) return false;
@@ -284,12 +283,12 @@ __global__ void __launch_bounds__(MmaCfg<D, MT, KP, NST>::THREADS, 1)
         const int flags = mtb.x & 0xff;
         if (flags & kTerm) {
             // the group that would take the next segment tells the epilogue
-            if ((int)(n_seg & 1) == grp && !hand_over(true, 0.f, 0.f) && lane == 0)
+            if ((int)(n_seg % C::NG) == grp && !hand_over(true, 0.f, 0.f) && lane == 0)
                 atomicOr(&p.err[blockIdx.x], (int)kErrTimeout);
             return;
         }
         if (flags & kFirst) {
-            own = (int)(n_seg & 1) == grp;
+            own = (int)(n_seg % C::NG) == grp;
             const int flags_q = mtb.x;
             cur_b = mta.x; cur_g = mta.y; leff = mta.w;
             cur_slot = mtb.y; cur_nseg = mtb.z; cur_first = mtb.w;
