@@ -365,16 +365,14 @@ __global__ void __launch_bounds__(kTokStreamThreads, kTokStreamCtas) tokens_stre
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_empty + 8 * s);
             if (++s == kTokStages) { s = 0; ph ^= 1; }
-            // the warp's best so far sets every lane's filter: an entry below
-            // it cannot be the maximum, and lanes that agree do not diverge
-            unsigned long long wp = kp, wr = kr;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                wp = umax64(wp, __shfl_xor_sync(0xffffffffu, wp, o));
-                wr = umax64(wr, __shfl_xor_sync(0xffffffffu, wr, o));
-            }
-            thr_p = __uint_as_float((uint32_t)(wp >> 32)) * kTokFilter;
-            thr_r = __uint_as_float((uint32_t)(wr >> 32)) * kTokFilter;
+            // the warp's best score so far sets every lane's filter: an entry
+            // below it cannot be the maximum, and lanes that agree do not
+            // diverge.  Scores are >= 0, so their bit patterns (a key's high
+            // word) order like the values: one integer max over the warp.
+            const uint32_t wp = __reduce_max_sync(0xffffffffu, (uint32_t)(kp >> 32));
+            const uint32_t wr = __reduce_max_sync(0xffffffffu, (uint32_t)(kr >> 32));
+            thr_p = __uint_as_float(wp) * kTokFilter;
+            thr_r = __uint_as_float(wr) * kTokFilter;
         }
         // the unit's best keys over the consumer threads
 #pragma unroll
