@@ -493,201 +493,285 @@ __global__ void __launch_bounds__(256, 2) magicdec_gather_kernel(const MdParams 
 }
 
 // ------------------------------------------------------------- MagicDec, fused
-// For up to 8 query heads per KV head the draft attention is computed where
-// the rows are read, in fp32 on the CUDA cores (4 FLOP per K/V byte: no
-// contraction worth the tensor cores).  One CTA per (sequence, KV head) pair
-// (a grid-stride loop over pairs): warp w of 4 takes 1/4 of the pair's visible
-// entries as the gather does (a batch of page lookups, then all the batch's
-// 16-byte K and V loads), turns and rounds the keys, and keeps for each of the
-// G query rows (turned by n - 1 and rounded, held by every row group of the
-// warp) a running maximum, sum and output in base 2; the warp's row groups
-// merge by shuffles, the four warps through shared memory in warp order, and
-// the CTA writes the G output rows.  A bad page, or a context length out of
-// range, gives NaN rows and SPIRE_DEVERR_CTX_LEN, as on the gather path.
-constexpr int kMfWarps = 4;        // one wave: 512 pairs fit as 4 CTAs per SM
-constexpr int kMfBatch = 3;      // row steps whose loads a lane issues together
+// For up to 8 query heads per KV head the draft attention is computed in one
+// kernel, one CTA of kMfWarps warps per (sequence, KV head) pair (a
+// grid-stride loop over pairs), on the warp-level tensor cores: the pair's
+// visible entries are taken kMfChunk at a time.  For a chunk, every thread
+// looks up one entry's page (all lookups in flight together), then the CTA
+// copies the chunk's K and V rows into shared memory with 16-byte
+// asynchronous copies (all in flight together; entries past the visible ones
+// and entries on a bad page are zero-filled), turns the window keys in place
+// (pairs d, d + D/2 of a row; every window entry moves by the same s - w0, so
+// one sine / cosine table per pair) and rounds them to bf16.  Warp w then owns
+// 16 entries of the chunk: S^T = K Q^T and O^T += V^T (P_hi + P_lo)^T with
+// the entries (and for PV the head dimensions) as the MMA's 16 rows and the
+// G <= 8 query heads (turned by n - 1, rounded to bf16, in shared memory) as
+// its 8 columns, and an online softmax in base 2 across chunks.  At the end
+// the warps' (O, m, l) rows meet in shared memory (over the K/V rows, no
+// longer needed) and are merged in warp order (deterministic).  A bad page,
+// or a context length out of range, gives NaN rows and SPIRE_DEVERR_CTX_LEN,
+// as on the gather path.
+constexpr int kMfWarps = 5;                    // 80-entry chunks: sink 1 + window 64 in one
+constexpr int kMfChunk = 16 * kMfWarps;
 
-template <int D, int GP>
-__global__ void __launch_bounds__(32 * kMfWarps, GP <= 4 ? 4 : 2)
-    magicdec_fused_kernel(const MdParams p) {
+template <int D>
+struct MfSmem {
+    static constexpr int HALF = kMfChunk * 128;          // one 64-column half of the K or V rows
+    static constexpr int KV = (D / 64) * HALF;
+    static constexpr int SCR = D + 8;                    // floats per hand-over row
+    static_assert(kMfWarps * 8 * SCR * 4 + kMfWarps * 8 * 8 <= 2 * KV,
+                  "the hand-over fits over the K/V rows");
+};
+
+template <int D>
+__global__ void __launch_bounds__(32 * kMfWarps, 4) magicdec_fused_kernel(const MdParams p) {
+    using M = MfSmem<D>;
+    __shared__ __align__(128) uint8_t kvs[2 * M::KV];    // K rows, then V rows (swizzled)
+    __shared__ __align__(128) uint8_t qs[(D / 64) * 1024];   // Q^T source: 8 rows, swizzled
     __shared__ uint64_t turn[64];
-    __shared__ float sm_o[kMfWarps][GP][D];
-    __shared__ float sm_ml[kMfWarps][GP][2];
-    __shared__ int sm_bad;
-    __shared__ uint32_t cta_err;
-    if (threadIdx.x < 64) turn[threadIdx.x] = p.fturn[threadIdx.x];
-    if (threadIdx.x == 0) cta_err = 0;
-    __syncthreads();
-    constexpr int LPR = D / 8, RPW = 32 / LPR, HL = LPR / 2;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int jl = lane % LPR, sub = lane / LPR;
-    const bool first_half = jl < HL;
-    const int d0 = 8 * (jl % HL);
+    __shared__ float tw_sn[D / 2], tw_cs[D / 2];         // window turn s - w0, per element
+    __shared__ float tq_sn[D / 2], tq_cs[D / 2];         // query turn n - 1, per element
+    __shared__ long long src[kMfChunk];                  // element offset of an entry's row
+    constexpr uint32_t FULL = 0xffffffffu;
+    constexpr int DT = D / 16;
+    const float NEG_INF = __int_as_float(0xff800000);
+    const float NANF = __int_as_float(0x7fc00000);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int gq = lane >> 2, tq = lane & 3;
+    const int ra = 2 * tq, rb = ra + 1;                  // query heads of this lane's columns
+    const uint32_t kbase = smem_u32(kvs), vbase = kbase + M::KV, qbase = smem_u32(qs);
+    float* const scr_o = reinterpret_cast<float*>(kvs);
+    float2* const scr_ml = reinterpret_cast<float2*>(kvs + kMfWarps * 8 * M::SCR * 4);
+    if (tid < 64) turn[tid] = p.fturn[tid];
+    uint32_t cta_err = 0;
     const long long pairs = (long long)p.B * p.Hkv;
     for (long long bg = blockIdx.x; bg < pairs; bg += gridDim.x) {
         const int g = (int)(bg % p.Hkv), b = (int)(bg / p.Hkv);
         const MdVisible v = md_visible(p, p.ctx_lens[b]);
-        const int rpp = (v.n + kMfWarps - 1) / kMfWarps;
-        const int c0 = warp * rpp, c1 = min(v.n, c0 + rpp);
-        if (threadIdx.x == 0) sm_bad = v.n == 0;
-        // the query rows of this KV head, turned by n - 1 and rounded to bf16
-        float qv[GP][8];
-        {
-            float sn[8], cs[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) { sn[e] = 0.f; cs[e] = 1.f; }
-            const bool turnq = p.rotate && v.n > 1;
-            if (turnq) md_lane_turn(turn, v.n - 1, d0, sn, cs);
-#pragma unroll
-            for (int h = 0; h < GP; ++h) {
-                uint4 x = make_uint4(0, 0, 0, 0);
-                if (h < p.G)
-                    x = *reinterpret_cast<const uint4*>(
-                        p.q + ((long long)b * p.Hq + (long long)g * p.G + h) * D + 8 * jl);
-                const uint4 w = shfl_xor_u4(x, HL);
-                const uint4 y = turnq ? md_turn_vec(x, w, sn, cs, first_half) : x;
-                const uint32_t a[4] = {y.x, y.y, y.z, y.w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    qv[h][2 * e] = bf16lo_to_f32(a[e]);
-                    qv[h][2 * e + 1] = bf16hi_to_f32(a[e]);
-                }
-            }
+        const bool turnw = p.rotate && v.s != v.w0, turnq = p.rotate && v.n > 1;
+        __syncthreads();                                 // turn[] loaded; the last pair is done
+        bool pbad = v.n == 0;                            // same in every thread
+        // an entry's page id (thread e < kMfChunk, entry c0 + e), or -1 past the
+        // visible entries; the load is issued here and consumed later
+        auto page_of = [&](int c0) -> int {
+            if (tid >= kMfChunk || c0 + tid >= v.n) return -1;
+            const int c = c0 + tid;
+            const int pos = c < v.s ? c : v.w0 + (c - v.s);
+            return p.block_table[(long long)b * p.max_pages + pos / kPage];
+        };
+        const int id0 = page_of(0);                      // in flight during the tables
+        // the per-element turns: of the window entries (s - w0) and of the query (n - 1)
+        for (int d = tid; d < D / 2; d += blockDim.x) {
+            float sn = 0.f, cs = 1.f, qsn = 0.f, qcs = 1.f;
+            if (turnw) md_sincos(turn, (long long)v.s - v.w0, d, &sn, &cs);
+            if (turnq) md_sincos(turn, (long long)v.n - 1, d, &qsn, &qcs);
+            tw_sn[d] = sn;
+            tw_cs[d] = cs;
+            tq_sn[d] = qsn;
+            tq_cs[d] = qcs;
         }
-        float wsn[8], wcs[8];
+        float o[DT][4];
+        float ma = NEG_INF, mb = NEG_INF, la = 0.f, lb = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) { wsn[e] = 0.f; wcs[e] = 1.f; }
-        if (p.rotate && v.s != v.w0) md_lane_turn(turn, (long long)v.s - v.w0, d0, wsn, wcs);
-        float m[GP], l[GP], o[GP][8];
-#pragma unroll
-        for (int h = 0; h < GP; ++h) {
-            m[h] = -INFINITY;
-            l[h] = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
-        }
-        bool bad = false;
-        for (int cb = c0; cb < c1; cb += RPW * kMfBatch) {
-            long long src[kMfBatch];
-            int row[kMfBatch];
-#pragma unroll
-            for (int i = 0; i < kMfBatch; ++i) {      // the entries' pages
-                const int c = cb + i * RPW + sub;
-                row[i] = -1;
-                src[i] = 0;
-                if (c < c1) {
+        for (int j = 0; j < DT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+        uint32_t qf[DT][2];
+        for (int c0 = 0; c0 < v.n; c0 += kMfChunk) {
+            const int ne = min(kMfChunk, v.n - c0);
+            const int id = c0 == 0 ? id0 : page_of(c0);
+            // ---- the chunk's pages (one lookup per thread, all in flight together)
+            int badpg = 0;
+            if (tid < kMfChunk) {
+                long long sr = -1;                       // -1: no row (zero-filled)
+                if (tid < ne) {
+                    const int c = c0 + tid;
                     const int pos = c < v.s ? c : v.w0 + (c - v.s);
-                    const int id = p.block_table[(long long)b * p.max_pages + pos / kPage];
-                    if (id >= 0 && id < p.num_pages) {
-                        row[i] = c;
-                        src[i] = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * D + 8 * jl;
-                    } else {
-                        bad = true;
-                    }
+                    if (id >= 0 && id < p.num_pages)
+                        sr = (((long long)id * p.Hkv + g) * kPage + pos % kPage) * D;
+                    else
+                        badpg = 1;
                 }
+                src[tid] = sr;
             }
-            uint4 kvk[kMfBatch], kvv[kMfBatch];
-#pragma unroll
-            for (int i = 0; i < kMfBatch; ++i) {      // all rows in flight together
-                if (row[i] >= 0) {
-                    kvk[i] = *reinterpret_cast<const uint4*>(p.k_cache + src[i]);
-                    kvv[i] = *reinterpret_cast<const uint4*>(p.v_cache + src[i]);
+            if (__syncthreads_or(badpg)) pbad = true;   // the tables and src[] are in place
+            // ---- K and V rows into shared memory (row e, 16-byte chunk ch at
+            // half ch / 8, row e, chunk (ch % 8) ^ (e % 8)); rows past the
+            // visible entries, or on a bad page, zero-filled
+            for (int i = tid; i < kMfChunk * (D / 8); i += blockDim.x) {
+                const int e = i / (D / 8), ch = i - e * (D / 8);
+                const uint32_t off = (ch >> 3) * M::HALF + e * 128 + (((ch & 7) ^ (e & 7)) << 4);
+                const long long sr = src[e];
+                if (sr >= 0) {
+                    cp_async16(kbase + off, p.k_cache + sr + 8 * ch);
+                    cp_async16(vbase + off, p.v_cache + sr + 8 * ch);
                 } else {
-                    kvk[i] = kvv[i] = make_uint4(0, 0, 0, 0);
+                    *reinterpret_cast<uint4*>(kvs + off) = make_uint4(0u, 0u, 0u, 0u);
+                    *reinterpret_cast<uint4*>(kvs + M::KV + off) = make_uint4(0u, 0u, 0u, 0u);
                 }
             }
-#pragma unroll
-            for (int i = 0; i < kMfBatch; ++i) {
-                const uint4 w = shfl_xor_u4(kvk[i], HL);
-                const bool valid = row[i] >= 0;
-                const bool sink = row[i] < v.s;
-                const uint4 kt = (sink || !p.rotate) ? kvk[i]
-                                                      : md_turn_vec(kvk[i], w, wsn, wcs, first_half);
-                const uint32_t ka[4] = {kt.x, kt.y, kt.z, kt.w};
-                const uint32_t va[4] = {kvv[i].x, kvv[i].y, kvv[i].z, kvv[i].w};
-                float kf[8], vf[8];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    kf[2 * e] = bf16lo_to_f32(ka[e]);
-                    kf[2 * e + 1] = bf16hi_to_f32(ka[e]);
-                    vf[2 * e] = bf16lo_to_f32(va[e]);
-                    vf[2 * e + 1] = bf16hi_to_f32(va[e]);
+            if (c0 == 0) {
+                // the query heads turned by n - 1, rounded to bf16, at their
+                // swizzled places (element d and d + D/2 of row h; rows >= G zero)
+                __nv_bfloat16* const q16 = reinterpret_cast<__nv_bfloat16*>(qs);
+                for (int i = tid; i < 8 * (D / 2); i += blockDim.x) {
+                    const int h = i / (D / 2), d = i - h * (D / 2);
+                    float x0 = 0.f, x1 = 0.f;
+                    if (h < p.G) {
+                        const __nv_bfloat16* qr =
+                            p.q + ((long long)b * p.Hq + (long long)g * p.G + h) * D;
+                        const float a0 = __bfloat162float(qr[d]), a1 = __bfloat162float(qr[d + D / 2]);
+                        x0 = turnq ? a0 * tq_cs[d] - a1 * tq_sn[d] : a0;
+                        x1 = turnq ? a1 * tq_cs[d] + a0 * tq_sn[d] : a1;
+                    }
+                    const int e0 = d, e1 = d + D / 2;
+                    q16[(e0 >> 6) * 512 + h * 64 + ((((e0 & 63) >> 3) ^ h) << 3) + (e0 & 7)] =
+                        __float2bfloat16_rn(x0);
+                    q16[(e1 >> 6) * 512 + h * 64 + ((((e1 & 63) >> 3) ^ h) << 3) + (e1 & 7)] =
+                        __float2bfloat16_rn(x1);
                 }
+            }
+            cp_async_wait_all();
+            __syncthreads();
+            // ---- window keys turned by s - w0 and rounded to bf16, in place
+            if (turnw) {
+                for (int i = tid; i < kMfChunk * (D / 16); i += blockDim.x) {
+                    const int e = i / (D / 16), ch = i - e * (D / 16), ch2 = ch + D / 16;
+                    if (e >= ne || c0 + e < v.s || src[e] < 0) continue;   // sinks keep their turn
+                    const uint32_t off1 = (ch >> 3) * M::HALF + e * 128 + (((ch & 7) ^ (e & 7)) << 4);
+                    const uint32_t off2 = (ch2 >> 3) * M::HALF + e * 128 + (((ch2 & 7) ^ (e & 7)) << 4);
+                    uint4* const p1 = reinterpret_cast<uint4*>(kvs + off1);
+                    uint4* const p2 = reinterpret_cast<uint4*>(kvs + off2);
+                    const uint4 a = *p1, w = *p2;
+                    const uint32_t av[4] = {a.x, a.y, a.z, a.w}, wv[4] = {w.x, w.y, w.z, w.w};
+                    uint32_t r1[4], r2[4];
 #pragma unroll
-                for (int h = 0; h < GP; ++h) {
-                    float sc = 0.f;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) sc = fmaf(qv[h][e], kf[e], sc);
-#pragma unroll
-                    for (int off = HL; off >= 1; off >>= 1)   // the row's LPR lanes
-                        sc += __shfl_xor_sync(0xffffffffu, sc, off);
-                    if (!valid) continue;
-                    const float s2 = sc * p.sl2;
-                    const float mn = fmaxf(m[h], s2);
-                    const float corr = exp2f(m[h] - mn), pe = exp2f(s2 - mn);
-                    m[h] = mn;
-                    l[h] = fmaf(l[h], corr, pe);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) o[h][e] = fmaf(o[h][e], corr, pe * vf[e]);
+                    for (int q = 0; q < 4; ++q) {
+                        const int d = 8 * ch + 2 * q;
+                        const float a0 = bf16lo_to_f32(av[q]), a1 = bf16hi_to_f32(av[q]);
+                        const float b0 = bf16lo_to_f32(wv[q]), b1 = bf16hi_to_f32(wv[q]);
+                        r1[q] = pack_bf16(a0 * tw_cs[d] - b0 * tw_sn[d], a1 * tw_cs[d + 1] - b1 * tw_sn[d + 1]);
+                        r2[q] = pack_bf16(b0 * tw_cs[d] + a0 * tw_sn[d], b1 * tw_cs[d + 1] + a1 * tw_sn[d + 1]);
+                    }
+                    *p1 = make_uint4(r1[0], r1[1], r1[2], r1[3]);
+                    *p2 = make_uint4(r2[0], r2[1], r2[2], r2[3]);
                 }
+                __syncthreads();
+            }
+            if (c0 == 0) {
+                // B = Q^T: lane (gq, tq) takes row gq, columns 2 tq, 2 tq + 1 of the
+                // 8x8 blocks at 16-byte chunks 2 ks and 2 ks + 1
+                const int qrow = lane & 7;
+#pragma unroll
+                for (int ks = 0; ks < DT; ks += 2) {
+                    const int chunk = 2 * ks + (lane >> 3);
+                    ldsm_x4(qf[ks][0], qf[ks][1], qf[ks + 1][0], qf[ks + 1][1],
+                            qbase + (chunk >> 3) * 1024 + qrow * 128 + (((chunk & 7) ^ qrow) << 4));
+                }
+            }
+            // ---- this warp's 16 entries: S^T = K Q^T (two accumulation chains)
+            const int wkey = 16 * warp;
+            const int krow = wkey + ((lane >> 3) & 1) * 8 + (lane & 7);
+            const int vrow = wkey + ((lane >> 4) << 3) + (lane & 7);
+            float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int ks = 0; ks < DT; ++ks) {
+                const int chunk = 2 * ks + (lane >> 4);
+                uint32_t a[4];
+                ldsm_x4(a[0], a[1], a[2], a[3],
+                        kbase + (chunk >> 3) * M::HALF + krow * 128 + (((chunk & 7) ^ (lane & 7)) << 4));
+                if (ks & 1) mma_bf16(s1, a, qf[ks][0], qf[ks][1]);
+                else        mma_bf16(s0, a, qf[ks][0], qf[ks][1]);
+            }
+            float s[4] = {s0[0] + s1[0], s0[1] + s1[1], s0[2] + s1[2], s0[3] + s1[3]};
+            if (wkey + gq >= ne) s[0] = s[1] = NEG_INF;          // past the visible entries
+            if (wkey + gq + 8 >= ne) s[2] = s[3] = NEG_INF;
+            // ---- online softmax (base 2); a head's 16 entries sit in the 8 lanes of its tq
+            float xa = fmaxf(s[0], s[2]), xb = fmaxf(s[1], s[3]);
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                xa = fmaxf(xa, __shfl_xor_sync(FULL, xa, off));
+                xb = fmaxf(xb, __shfl_xor_sync(FULL, xb, off));
+            }
+            const float mna = fmaxf(ma, xa * p.sl2), mnb = fmaxf(mb, xb * p.sl2);
+            const float mra = (mna == NEG_INF) ? 0.f : mna;
+            const float mrb = (mnb == NEG_INF) ? 0.f : mnb;
+            const float aa = ex2(ma - mra), ab = ex2(mb - mrb);
+            ma = mna; mb = mnb;
+            s[0] = ex2(fmaf(s[0], p.sl2, -mra));
+            s[1] = ex2(fmaf(s[1], p.sl2, -mrb));
+            s[2] = ex2(fmaf(s[2], p.sl2, -mra));
+            s[3] = ex2(fmaf(s[3], p.sl2, -mrb));
+            la = la * aa + (s[0] + s[2]);
+            lb = lb * ab + (s[1] + s[3]);
+#pragma unroll
+            for (int j = 0; j < DT; ++j) {
+                o[j][0] *= aa; o[j][1] *= ab;
+                o[j][2] *= aa; o[j][3] *= ab;
+            }
+            // ---- O^T += V^T (P_hi + P_lo)^T, P^T moved into the B layout
+            const uint32_t h0 = pack_bf16(s[0], s[1]), h1 = pack_bf16(s[2], s[3]);
+            const uint32_t l0 = pack_bf16(s[0] - bf16lo_to_f32(h0), s[1] - bf16hi_to_f32(h0));
+            const uint32_t l1 = pack_bf16(s[2] - bf16lo_to_f32(h1), s[3] - bf16hi_to_f32(h1));
+            const uint32_t bh0 = movm_trans(h0), bh1 = movm_trans(h1);
+            const uint32_t bl0 = movm_trans(l0), bl1 = movm_trans(l1);
+#pragma unroll
+            for (int j = 0; j < DT; ++j) {
+                const int chunk = 2 * j + ((lane >> 3) & 1);
+                uint32_t a[4];
+                ldsm_x4_trans(a[0], a[1], a[2], a[3],
+                              vbase + (chunk >> 3) * M::HALF + vrow * 128 + (((chunk & 7) ^ (lane & 7)) << 4));
+                mma_bf16(o[j], a, bh0, bh1);
+                mma_bf16(o[j], a, bl0, bl1);
+            }
+            __syncthreads();                             // the rows are read: next chunk, or hand-over
+        }
+        // ---- the warps' rows meet in shared memory, merged in warp order
+        float lta = la, ltb = lb;
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            lta += __shfl_xor_sync(FULL, lta, off);
+            ltb += __shfl_xor_sync(FULL, ltb, off);
+        }
+        float* const so = scr_o + warp * 8 * M::SCR;
+        if (ra < p.G) {
+#pragma unroll
+            for (int j = 0; j < DT; ++j) {
+                so[ra * M::SCR + 16 * j + gq] = o[j][0];
+                so[ra * M::SCR + 16 * j + gq + 8] = o[j][2];
             }
         }
-        // the warp's row groups hold different entries: merge them
+        if (rb < p.G) {
 #pragma unroll
-        for (int off = LPR; off < 32; off <<= 1) {
-#pragma unroll
-            for (int h = 0; h < GP; ++h) {
-                const float m2 = __shfl_xor_sync(0xffffffffu, m[h], off);
-                const float l2 = __shfl_xor_sync(0xffffffffu, l[h], off);
-                const float mn = fmaxf(m[h], m2);
-                const float c1s = mn == -INFINITY ? 0.f : exp2f(m[h] - mn);
-                const float c2s = mn == -INFINITY ? 0.f : exp2f(m2 - mn);
-                l[h] = l[h] * c1s + l2 * c2s;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float o2 = __shfl_xor_sync(0xffffffffu, o[h][e], off);
-                    o[h][e] = o[h][e] * c1s + o2 * c2s;
-                }
-                m[h] = mn;
+            for (int j = 0; j < DT; ++j) {
+                so[rb * M::SCR + 16 * j + gq] = o[j][1];
+                so[rb * M::SCR + 16 * j + gq + 8] = o[j][3];
             }
         }
-        if (__any_sync(0xffffffffu, bad) && lane == 0) sm_bad = 1;
-        if (sub == 0) {
-#pragma unroll
-            for (int h = 0; h < GP; ++h) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) sm_o[warp][h][8 * jl + e] = o[h][e];
-                if (jl == 0) {
-                    sm_ml[warp][h][0] = m[h];
-                    sm_ml[warp][h][1] = l[h];
-                }
-            }
+        if (gq == 0) {
+            scr_ml[warp * 8 + ra] = make_float2(ma, lta);
+            scr_ml[warp * 8 + rb] = make_float2(mb, ltb);
         }
         __syncthreads();
-        // the warps' results, in warp order, for the G rows
-        const bool pbad = sm_bad != 0;
-        if (pbad && threadIdx.x == 0) cta_err |= kErrCtxLen;
-        for (int i = threadIdx.x; i < p.G * D; i += blockDim.x) {
-            const int h = i / D, d = i % D;
-            float M = -INFINITY;
+        if (pbad) cta_err |= kErrCtxLen;
+        for (int i = tid; i < p.G * D; i += blockDim.x) {
+            const int h = i / D, d = i - h * D;
+            float Mx = NEG_INF;
 #pragma unroll
-            for (int w = 0; w < kMfWarps; ++w) M = fmaxf(M, sm_ml[w][h][0]);
+            for (int w = 0; w < kMfWarps; ++w) Mx = fmaxf(Mx, scr_ml[w * 8 + h].x);
+            const float Mr = (Mx == NEG_INF) ? 0.f : Mx;
             float L = 0.f, O = 0.f;
 #pragma unroll
             for (int w = 0; w < kMfWarps; ++w) {
-                const float mw = sm_ml[w][h][0];
-                if (mw == -INFINITY) continue;
-                const float sc = exp2f(mw - M);
-                L = fmaf(sm_ml[w][h][1], sc, L);
-                O = fmaf(sm_o[w][h][d], sc, O);
+                const float2 ml = scr_ml[w * 8 + h];
+                const float sc = ex2(ml.x - Mr);
+                L = fmaf(ml.y, sc, L);
+                O = fmaf(scr_o[(w * 8 + h) * M::SCR + d], sc, O);
             }
             p.out[((long long)b * p.Hq + (long long)g * p.G + h) * D + d] =
-                (pbad || !(L > 0.f)) ? NAN : O / L;
+                (pbad || !(L > 0.f)) ? NANF : O / L;
         }
-        __syncthreads();                         // shared memory is reused by the next pair
     }
     // one error word per CTA: every CTA writes its own, nothing needs clearing
-    if (threadIdx.x == 0) {
+    if (tid == 0) {
         p.err[blockIdx.x] = (int32_t)cta_err;
         if (blockIdx.x == 0) p.header[0] = (int32_t)gridDim.x;
     }
@@ -969,12 +1053,9 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
         mp.out = out;
         const long long pairs = (long long)mp.B * mp.Hkv;
         const long long fblocks = pairs < kMaxCtas ? pairs : kMaxCtas;   // one error word each
-        void (*fk)(MdParams) = nullptr;
-#define SPIRE_MD_CASE(DD, GG) \
-    if (desc->head_dim == DD && gp == GG) fk = magicdec_fused_kernel<DD, GG>;
-        SPIRE_MD_CASE(64, 1) SPIRE_MD_CASE(64, 2) SPIRE_MD_CASE(64, 4) SPIRE_MD_CASE(64, 8)
-        SPIRE_MD_CASE(128, 1) SPIRE_MD_CASE(128, 2) SPIRE_MD_CASE(128, 4) SPIRE_MD_CASE(128, 8)
-#undef SPIRE_MD_CASE
+        void (*fk)(MdParams) = desc->head_dim == 128 ? magicdec_fused_kernel<128>
+                               : desc->head_dim == 64  ? magicdec_fused_kernel<64>
+                                                       : nullptr;
         if (!fk) return SPIRE_ERR_UNSUPPORTED;
         fk<<<(unsigned)fblocks, 32 * kMfWarps, 0, s>>>(mp);   // after all prior work
         return cudaGetLastError() == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;

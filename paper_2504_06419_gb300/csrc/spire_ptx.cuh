@@ -199,6 +199,16 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1, uint32
                  : "r"(addr));
 }
 
+// 16-byte asynchronous copy global -> shared (both 16-byte aligned), bypassing
+// L1; completion by cp_async_wait_all.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 // Transpose of an 8x8 b16 matrix held one 32-bit pair per lane (lane l holds
 // row l/4, columns 2(l%4) and 2(l%4)+1); returns the same lane's pair of the
 // transposed matrix.

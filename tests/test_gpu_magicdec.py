@@ -37,6 +37,8 @@ CASES = [
     ("ragged_sink4_win128", [5, 63, 64, 129, 5000, 70000], 8, 2, 128, 4, 128, 10000.0),
     ("window_covers_context", [10, 100, 200], 4, 2, 64, 4, 256, 10000.0),
     ("no_rotation", [300, 301, 302], 8, 8, 64, 2, 30, 0.0),
+    ("g8_d128", [4000, 77, 9000], 64, 8, 128, 1, 64, 10000.0),
+    ("g3_two_chunks", [500, 1500, 90], 6, 2, 128, 2, 100, 10000.0),
     # 64 query heads per KV head: the draft attention runs on the tcgen05 kernel
     ("g64_tcgen05", [100, 3000, 40], 64, 1, 64, 1, 64, 10000.0),
 ]
