@@ -437,6 +437,18 @@ static inline SPIRE_HOST_DEVICE int64_t spire_draft_slot_inline(int64_t pos, int
 SPIRE_API int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window);
 
 /*
+ * spire_test_draft_slots -- a test hook; the paper has no counterpart.  One
+ * kernel launch that writes spire_draft_slot_inline(p, n_sink, window),
+ * evaluated on the device, to out[p] for p = 0 .. n-1 (int64, device memory,
+ * 8-byte aligned), so that tests can hold the device evaluation of the inline
+ * helper (the one the cache-writing kernel uses) against the host's.
+ * Asynchronous on `stream`.  Returns SPIRE_ERR_INVALID_ARG for n < 0 or a null
+ * or misaligned out (n = 0 is a no-op).
+ */
+SPIRE_API spire_status spire_test_draft_slots(int64_t *out, int64_t n, int32_t n_sink,
+                                              int32_t window, void *stream);
+
+/*
  * spire_get_device_error -- copy the device error word of the most recent
  * call that used `workspace` into *code_out (0 = no error, else an OR of
  * SPIRE_DEVERR_* bits).  Synchronises `stream`.

@@ -30,7 +30,7 @@ from ._lib import (SpireError, make_append_desc, make_desc, spire_draft_slot,
                    spire_draft_sparse_attention, spire_draft_workspace_bytes,
                    spire_feedback_append, spire_feedback_append_workspace_bytes,
                    spire_get_cta_times, spire_get_device_error, spire_magicdec_attention,
-                   spire_stream_read, spire_test_stall_next_call,
+                   spire_stream_read, spire_test_draft_slots, spire_test_stall_next_call,
                    spire_magicdec_workspace_bytes, spire_status_string, spire_verify_attention,
                    spire_verify_attention_noalloc, spire_verify_tokens,
                    spire_verify_tokens_workspace_bytes, spire_verify_workspace_bytes)
@@ -42,7 +42,8 @@ __all__ = [
     "spire_verify_tokens_workspace_bytes", "verify_tokens", "spire_magicdec_attention",
     "spire_magicdec_workspace_bytes", "magicdec_attention",
     "spire_verify_workspace_bytes", "spire_draft_workspace_bytes", "spire_draft_slot",
-    "spire_get_device_error", "spire_get_cta_times", "spire_stream_read", "spire_test_stall_next_call", "spire_status_string",
+    "spire_get_device_error", "spire_get_cta_times", "spire_stream_read", "spire_test_draft_slots",
+    "spire_test_stall_next_call", "spire_status_string",
     "verify_attention",
     "draft_attention",
     "verify_desc", "draft_desc",

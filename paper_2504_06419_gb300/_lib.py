@@ -46,6 +46,7 @@ EXPORTED = (
     "spire_get_cta_times",
     "spire_stream_read",
     "spire_test_stall_next_call",
+    "spire_test_draft_slots",
     "spire_status_string",
 )
 
@@ -125,6 +126,8 @@ def _load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.spire_stream_read.argtypes = [P, SZ, P]
     lib.spire_test_stall_next_call.restype = ctypes.c_int
     lib.spire_test_stall_next_call.argtypes = [I32]
+    lib.spire_test_draft_slots.restype = ctypes.c_int
+    lib.spire_test_draft_slots.argtypes = [P, ctypes.c_int64, I32, I32, P]
     lib.spire_status_string.restype = ctypes.c_char_p
     lib.spire_status_string.argtypes = [ctypes.c_int]
     return lib
@@ -264,6 +267,13 @@ def spire_stream_read(src, nbytes, stream=None) -> int:
     """One launch that only reads nbytes at src (the floor of a call that
     moves that many bytes); see include/spire.h."""
     return int(LIB.spire_stream_read(_ptr(src), int(nbytes), _stream(stream, src)))
+
+
+def spire_test_draft_slots(out, n, n_sink, window, stream=None) -> int:
+    """Test hook: the device evaluation of the slot helper for p = 0..n-1
+    into out (int64); see include/spire.h."""
+    return int(LIB.spire_test_draft_slots(_ptr(out), int(n), int(n_sink), int(window),
+                                          _stream(stream, out)))
 
 
 def spire_test_stall_next_call(pair) -> int:

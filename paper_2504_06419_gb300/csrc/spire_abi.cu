@@ -777,6 +777,13 @@ __global__ void __launch_bounds__(32 * kMfWarps, 4) magicdec_fused_kernel(const 
     }
 }
 
+// spire_test_draft_slots: the inline slot helper evaluated on the device
+__global__ void draft_slots_kernel(int64_t* out, long long n, int32_t n_sink, int32_t window) {
+    for (long long p = blockIdx.x * (long long)blockDim.x + threadIdx.x; p < n;
+         p += (long long)gridDim.x * blockDim.x)
+        out[p] = spire_draft_slot_inline(p, n_sink, window);
+}
+
 struct MdLayout {
     size_t draft, kv, q, nvis, total;
 };
@@ -1077,6 +1084,17 @@ spire_status spire_magicdec_attention(const void* q, const void* k_cache, const 
 
 int64_t spire_draft_slot(int64_t pos, int32_t n_sink, int32_t window) {
     return spire_draft_slot_inline(pos, n_sink, window);
+}
+
+spire_status spire_test_draft_slots(int64_t* out, int64_t n, int32_t n_sink, int32_t window,
+                                    void* stream) {
+    if (n < 0) return SPIRE_ERR_INVALID_ARG;
+    if (n == 0) return SPIRE_OK;
+    if (!out || !aligned(out, 8)) return SPIRE_ERR_INVALID_ARG;
+    const long long blocks = (n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096;
+    draft_slots_kernel<<<(unsigned)blocks, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        out, (long long)n, n_sink, window);
+    return cudaGetLastError() == cudaSuccess ? SPIRE_OK : SPIRE_ERR_CUDA;
 }
 
 spire_status spire_get_device_error(const void* workspace, int32_t* code_out, void* stream) {

@@ -32,7 +32,7 @@ def test_header_declares_the_boundary():
         "spire_verify_tokens_workspace_bytes", "spire_verify_tokens",
         "spire_magicdec_workspace_bytes", "spire_magicdec_attention",
         "spire_get_device_error", "spire_get_cta_times", "spire_stream_read",
-        "spire_test_stall_next_call", "spire_status_string"]), names
+        "spire_test_draft_slots", "spire_test_stall_next_call", "spire_status_string"]), names
 
 
 def test_library_exports_every_declared_symbol(spire):
@@ -262,6 +262,15 @@ def test_stream_read_host_checks(spire):
     assert spire.spire_stream_read(None, 16, 0) == 1
     assert spire.spire_stream_read(1 << 20, 8, 0) == 1
     assert spire.spire_stream_read((1 << 20) + 8, 16, 0) == 1
+
+
+def test_draft_slots_hook_host_checks(spire):
+    # n = 0 is a no-op; a negative n, a null or a misaligned output is refused
+    # before anything is launched
+    assert spire.spire_test_draft_slots(None, 0, 4, 64, 0) == 0
+    assert spire.spire_test_draft_slots(None, 10, 4, 64, 0) == 1
+    assert spire.spire_test_draft_slots(1 << 20, -1, 4, 64, 0) == 1
+    assert spire.spire_test_draft_slots((1 << 20) + 4, 10, 4, 64, 0) == 1
 
 
 def test_stall_hook_host_checks(spire):
