@@ -286,6 +286,41 @@ def verify_config_entry(spire, name, dev, stream, flush, args, hbm_peak, max_seq
              "traffic": dram_traffic("verify:%s" % name), "clocks": clocks}
     del vi, ws, out
     torch.cuda.empty_cache()
+
+    # the round's k draft steps on this workload's bounded cache (step j sees
+    # t = L - k + j entries), each call timed like the verify call, and the
+    # speculation-round attention rate of one layer: B (k+1) / (t_verify + sum t_draft)
+    S = cfg.n_sink + cfg.window
+    di = wl.make_draft(wl.draft_ctx_for_step(L, k, 0), Hq, Hkv, D, cfg.n_sink, cfg.window,
+                       seed=cfg.seed + 17, device=dev)
+    ctxs = [torch.from_numpy(wl.draft_ctx_for_step(L, k, j)).to(dev) for j in range(k)]
+    ddesc = spire.draft_desc(di.q, di.kv)
+    dws = torch.empty(spire.spire_draft_workspace_bytes(ddesc, cfg.n_sink, cfg.window),
+                      dtype=torch.uint8, device=dev)
+    dout = torch.empty(di.q.shape, dtype=torch.float32, device=dev)
+
+    def draft_call(j):
+        st = spire.spire_draft_sparse_attention(di.q, di.kv, ctxs[j], cfg.n_sink, cfg.window,
+                                                ddesc, dout, dws, dws.numel(), sptr)
+        if st:
+            raise spire.SpireError(st, "spire_draft_sparse_attention (%s)" % name)
+
+    for _ in range(args.warmup):
+        for j in range(k):
+            draft_call(j)
+    torch.cuda.synchronize(dev)
+    if spire.spire_get_device_error(dws, stream):
+        raise RuntimeError("device error word set by the %s draft call" % name)
+    d_ms = sum(reduce_max([event_ms(lambda: draft_call(j), n, flush, stream)], dist, dev)[0]
+               for j in range(k))
+    db = sum(draft_bytes(wl.draft_ctx_for_step(L, k, j), S, Hq, Hkv, D) for j in range(k))
+    entry["draft"] = {"steps": k, "ms_total": d_ms, "algorithmic_bytes": db,
+                      "gbs": db / (d_ms * 1e-3) / 1e9,
+                      "frac": db / (d_ms * 1e-3) / 1e9 / hbm_peak,
+                      "cache_gb": di.kv.numel() * 2 / 1e9}
+    entry["round_tokens_per_s"] = B * (k + 1) / ((ms + d_ms) * 1e-3)
+    del di, ctxs, dws, dout
+    torch.cuda.empty_cache()
     return entry
 
 
