@@ -111,15 +111,19 @@ class ClockSampler:
 
 def source_sha16():
     """Hash of the device code and launch configuration (the .cuh kernels and
-    spire_launch.h): the files whose change invalidates the ncu counters."""
+    spire_launch.h, comments and blank lines left out): the code whose change
+    invalidates the ncu counters."""
     import hashlib
+    import re
     d = os.path.join(ROOT, "paper_2504_06419_gb300", "csrc")
     h = hashlib.sha256()
     for f in sorted(os.listdir(d)):
         if f.endswith(".cuh") or f == "spire_launch.h":
             h.update(f.encode())
-            with open(os.path.join(d, f), "rb") as fh:
-                h.update(fh.read())
+            with open(os.path.join(d, f)) as fh:
+                src = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)
+            lines = (re.sub(r"//.*", "", ln).rstrip() for ln in src.splitlines())
+            h.update("\n".join(ln for ln in lines if ln).encode())
     return h.hexdigest()[:16]
 
 

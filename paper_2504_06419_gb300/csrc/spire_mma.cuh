@@ -2,23 +2,26 @@
 // (mma.sync m16n8k16, bf16 in / fp32 accumulate).
 //
 // Roles in a CTA (one CTA per SM):
-//   warp NW (producer)  lane 0 walks the CTA's tile range, translates pages
+//   warp NCW (producer) lane 0 walks the CTA's tile range, translates pages
 //                       through the block table, and streams each K and V
 //                       tile with TMA (64 keys x D, 128-byte swizzle) into
 //                       an NST-deep ring of shared-memory stages.
-//   warps 0..NW-1       consumer warp w owns key slice w (64 / KP = 16 keys
+//   warps 0..NCW-1      NG = 2 groups of NW = 4 consumer warps; the groups
+//                       take turns by segment of the walk, so each SM
+//                       sub-partition runs two independent consumer chains.
+//                       Consumer warp w of a group owns key slice w (16 keys
 //                       of every tile).  It keeps Q^T in registers for the
 //                       current pair, runs S^T = K Q^T and O^T += V^T P^T on
 //                       the tensor cores (keys and head dimensions as the
 //                       MMA's 16 rows, the pair's query rows as its 8
 //                       columns) and an fp32 online softmax in base 2.
-//   warp NW+1 (epilogue) at the end of a pair's segment the consumers only
-//                       hand their (O, m, l) rows to one of two shared-memory
-//                       buffers and go on with the next segment; this warp
-//                       merges the KP key slices and writes the result to the
-//                       output, or to a partial slot that the last-arriving
-//                       CTA merges (see spire_common.cuh), publishing with a
-//                       fence and an atomic, off the consumers' path.
+//   warp NCW+1 (epilogue) at the end of a pair's segment the owning group only
+//                       hands its (O, m, l) rows to one of two shared-memory
+//                       buffers and goes on; this warp merges the NW key
+//                       slices and writes the result to the output, or to a
+//                       partial slot that the last-arriving CTA merges (see
+//                       spire_common.cuh), publishing with a fence and an
+//                       atomic, off the consumers' path.
 // The kernel serves pairs of at most 8 query rows (the MMA's N = 8), so a
 // buffer holds 8 rows per consumer warp.
 //
