@@ -36,6 +36,7 @@ VERIFY_CASES = [
     ([300, 1200], 16, 4, 1, 128),              # 68 rows
     ([500, 90], 64, 1, 1, 128),                # 65 rows, G = 1
     ([2000, 80], 8, 64, 8, 64),                # 72 rows at D = 64
+    ([900, 300, 4100], 2, 6, 3, 128),          # 6 rows per KV head (warp-MMA kernel)
 ]
 
 
@@ -172,6 +173,8 @@ DRAFT_CASES = [
     ([1, 5, 6, 7, 100], 8, 8, 128, 1, 4),         # S = 5 < one tile
     ([3, 300, 5000], 64, 8, 128, 32, 2048),       # G = 8
     ([10, 20, 4000], 16, 2, 64, 0, 100),          # no sinks
+    ([700, 70, 3000], 24, 8, 128, 16, 512),       # G = 3: an odd row count
+    ([50, 900, 1300], 14, 2, 128, 4, 200),        # G = 7
 ]
 
 
