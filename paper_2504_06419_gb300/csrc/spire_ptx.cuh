@@ -332,6 +332,22 @@ __device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t s_desc
                  : "memory");
 }
 
+// 32 rows x 16 bytes from shared memory into the same columns of all four
+// lane quarters of tensor memory (rows r -> lanes r, 32 + r, 64 + r, 96 + r).
+__device__ __forceinline__ void tmem_cp_32x128b_x4(uint32_t taddr, uint64_t s_desc) {
+    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(s_desc)
+                 : "memory");
+}
+
+// 64 rows x 16 bytes from shared memory into tensor memory twice: rows 0..31
+// to lane quarters 0 and 2, rows 32..63 to quarters 1 and 3 (rows r -> lanes
+// r and 64 + r).
+__device__ __forceinline__ void tmem_cp_64x128b_x2(uint32_t taddr, uint64_t s_desc) {
+    asm volatile("tcgen05.cp.cta_group::1.64x128b.warpx2::02_13 [%0], %1;" ::"r"(taddr),
+                 "l"(s_desc)
+                 : "memory");
+}
+
 // Arrive on an mbarrier once every tcgen05 operation this thread issued so far
 // has completed.
 __device__ __forceinline__ void umma_commit(uint32_t bar) {

@@ -53,7 +53,10 @@ struct TcCfg {
     static constexpr int THREADS = 224;
     static constexpr int TILE = kPage * D * 2;     // one K (or V) tile
     static constexpr int STAGE = 2 * TILE;
-    static constexpr int QHALF = 128 * 128;        // 128 rows x 64 columns of bf16
+    // one copy of the query rows in shared memory (128 / NC rows of 64 columns
+    // per half); tcgen05.cp replicates it into the NC copies in tensor memory
+    static constexpr int QROWS = 128 / NC;
+    static constexpr int QHALF = QROWS * 128;
     static constexpr int QBUF = (D / 64) * QHALF;
     static constexpr int KW = kPage / NC;          // keys of a tile per copy
     static constexpr int RB = 4 / NC;              // 32-row blocks per copy
@@ -61,7 +64,7 @@ struct TcCfg {
     static constexpr int SCR_LD = 33;              // floats per scratch row (32 + pad)
     static constexpr int OFF_Q = NST * STAGE;
     static constexpr int OFF_SCR = OFF_Q + QBUF;   // one Q buffer: copied to TMEM at once
-    static constexpr int OFF_ML = OFF_SCR + 2 * SCR_ROWS * SCR_LD * 4;
+    static constexpr int OFF_ML = OFF_SCR + SCR_ROWS * SCR_LD * 4;
     static constexpr int OFF_META = OFF_ML + 128 * 8;
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
     static constexpr int OFF_MISC = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16;
@@ -71,7 +74,7 @@ struct TcCfg {
     static constexpr uint32_t TMEM_COLS = 512;
     static constexpr int S_COL = 0, O_COL = 128, P_COL = 256, Q_COL = 384;
     static_assert(NC == 1 || NC == 2 || NC == 4, "1, 2 or 4 query copies");
-    static_assert(STAGE % 1024 == 0 && OFF_Q % 1024 == 0,
+    static_assert(STAGE % 1024 == 0 && OFF_Q % 1024 == 0 && QHALF % 1024 == 0,
                   "swizzled regions must be 1024-byte aligned");
     static_assert(O_COL + D <= P_COL && Q_COL + D <= (int)TMEM_COLS, "tensor memory budget");
 };
@@ -148,8 +151,9 @@ __global__ void __launch_bounds__(224, 1)
     if (warp == 0) {
         // ------------------------------------------------------ producer
         if (lane == 0) {
+            // one copy of the query rows: tcgen05.cp replicates them
             const ProducerSmem ps{base, qsm, (uint32_t)C::QHALF, meta, bar_full,
-                                  bar_empty, bar_qfull, bar_qempty, NC, 128 / NC, 1, false};
+                                  bar_empty, bar_qfull, bar_qempty, 1, 0, 1, false};
             err |= produce<D, NST, kStall>(p, *sh, &tmap_k, &tmap_v, &tmap_q, ps);
         }
     } else if (warp == 1) {
@@ -175,11 +179,23 @@ __global__ void __launch_bounds__(224, 1)
                         cq ^= 1;
                         tc_fence_after();
                         const uint32_t qaddr = qsm;
+                        const uint32_t qdst = tmem + C::Q_COL + qb * (D / 2);
+                        if constexpr (NC == 1) {
 #pragma unroll
-                        for (int ks = 0; ks < D / 16; ++ks)
-                            tmem_cp_128x256b(tmem + C::Q_COL + qb * (D / 2) + ks * 8,
-                                             sdesc_sw128(qaddr + (ks >> 2) * C::QHALF + (ks & 3) * 32,
-                                                         16, 1024));
+                            for (int ks = 0; ks < D / 16; ++ks)   // 32 bytes of each row
+                                tmem_cp_128x256b(qdst + ks * 8,
+                                                 sdesc_sw128(qaddr + (ks >> 2) * C::QHALF + (ks & 3) * 32,
+                                                             16, 1024));
+                        } else {
+                            // 16 bytes of each row at a time, into every copy at once
+#pragma unroll
+                            for (int j = 0; j < D / 8; ++j) {
+                                const uint64_t sd =
+                                    sdesc_sw128(qaddr + (j >> 3) * C::QHALF + (j & 7) * 16, 16, 1024);
+                                if constexpr (NC == 4) tmem_cp_32x128b_x4(qdst + j * 4, sd);
+                                else                   tmem_cp_64x128b_x2(qdst + j * 4, sd);
+                            }
+                        }
                         umma_commit(bar_qempty);   // smem buffer free once copied
                     }
                 }
@@ -514,8 +530,9 @@ __global__ void __launch_bounds__(224, 1)
                         tmem_ld32(trow + C::O_COL + 32 * c, ov);
                         tmem_wait_ld();
                     }
-                    float* const sc = scr + (c & 1) * C::SCR_ROWS * C::SCR_LD;
+                    float* const sc = scr;           // one buffer: read before the next chunk
                     if (NC > 1) {
+                        if (c > 0 && !grp_sync()) { ok = false; break; }   // copy 0 read the last
                         if (copy > 0 && active) {
                             float* const row = sc + (tl - 32 * C::RB) * C::SCR_LD;
 #pragma unroll
