@@ -61,10 +61,12 @@ struct TcCfg {
     static constexpr int KW = kPage / NC;          // keys of a tile per copy
     static constexpr int RB = 4 / NC;              // 32-row blocks per copy
     static constexpr int SCR_ROWS = (NC - 1) * 32 * RB;   // rows of copies 1 .. NC-1
-    static constexpr int SCR_LD = 33;              // floats per scratch row (32 + pad)
+    // floats per scratch row; 16-byte chunk q of row t sits at q ^ (t % 8), so
+    // the 8 lanes of a 16-byte access phase, one row each, never share a bank
+    static constexpr int SCR_LD = 32;
     static constexpr int OFF_Q = NST * STAGE;
     static constexpr int OFF_SCR = OFF_Q + QBUF;   // one Q buffer: copied to TMEM at once
-    static constexpr int OFF_ML = OFF_SCR + SCR_ROWS * SCR_LD * 4;
+    static constexpr int OFF_ML = OFF_SCR + 2 * SCR_ROWS * SCR_LD * 4;   // two scratch buffers
     static constexpr int OFF_META = OFF_ML + 128 * 8;
     static constexpr int OFF_SCHED = OFF_META + NST * 32;
     static constexpr int OFF_MISC = OFF_SCHED + ((int(sizeof(SchedShared)) + 15) / 16) * 16;
@@ -530,24 +532,33 @@ __global__ void __launch_bounds__(224, 1)
                         tmem_ld32(trow + C::O_COL + 32 * c, ov);
                         tmem_wait_ld();
                     }
-                    float* const sc = scr;           // one buffer: read before the next chunk
+                    float* const sc = scr + (c & 1) * C::SCR_ROWS * C::SCR_LD;
                     if (NC > 1) {
-                        if (c > 0 && !grp_sync()) { ok = false; break; }   // copy 0 read the last
                         if (copy > 0 && active) {
-                            float* const row = sc + (tl - 32 * C::RB) * C::SCR_LD;
+                            float4* const row =
+                                reinterpret_cast<float4*>(sc + (tl - 32 * C::RB) * C::SCR_LD);
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) row[j] = ov[j] * wgt;
+                            for (int q = 0; q < 8; ++q)
+                                row[q ^ (lane & 7)] = make_float4(ov[4 * q] * wgt, ov[4 * q + 1] * wgt,
+                                                                  ov[4 * q + 2] * wgt, ov[4 * q + 3] * wgt);
                         }
                         if (!grp_sync()) { ok = false; break; }
                     }
                     if (dst) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            float acc = ov[j] * wgt;
+                        for (int q = 0; q < 8; ++q) {
+                            float4 acc = make_float4(ov[4 * q] * wgt, ov[4 * q + 1] * wgt,
+                                                     ov[4 * q + 2] * wgt, ov[4 * q + 3] * wgt);
 #pragma unroll
-                            for (int cc = 1; cc < NC; ++cc)
-                                acc += sc[(32 * C::RB * (cc - 1) + r) * C::SCR_LD + j];
-                            ov[j] = acc * inv;
+                            for (int cc = 1; cc < NC; ++cc) {
+                                const float4 o2 = reinterpret_cast<const float4*>(
+                                    sc + (32 * C::RB * (cc - 1) + r) * C::SCR_LD)[q ^ (lane & 7)];
+                                acc.x += o2.x; acc.y += o2.y; acc.z += o2.z; acc.w += o2.w;
+                            }
+                            ov[4 * q] = acc.x * inv;
+                            ov[4 * q + 1] = acc.y * inv;
+                            ov[4 * q + 2] = acc.z * inv;
+                            ov[4 * q + 3] = acc.w * inv;
                         }
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
