@@ -30,12 +30,17 @@ VERIFY_CASES = [
     ([4100, 70, 1000, 2049], 4, 32, 8, 128),   # splits + ragged
     ([17, 33], 15, 8, 1, 128),                 # 128 rows per KV head (maximum)
     ([100, 260], 2, 6, 2, 128),                # G = 3 (rows not a multiple of 8)
-    # just past 64 rows per KV head (one query copy)
+    # past 64 rows per KV head (one query copy)
     ([4100, 70, 1000, 2049, 300], 8, 64, 8, 128),   # 72 rows, many split pairs
     ([700, 64, 1500], 32, 2, 1, 128),          # 66 rows
     ([300, 1200], 16, 4, 1, 128),              # 68 rows
     ([500, 90], 64, 1, 1, 128),                # 65 rows, G = 1
     ([2000, 80], 8, 64, 8, 64),                # 72 rows at D = 64
+    ([1000, 129, 64], 9, 64, 8, 128),          # 80 rows
+    ([300, 1500, 65], 4, 32, 2, 128),          # 80 rows, G = 16
+    ([777, 2100], 4, 32, 2, 64),               # 80 rows, G = 16, D = 64
+    ([800, 333], 13, 10, 2, 128),              # 70 rows, G = 5
+    ([500, 70, 3000], 11, 16, 2, 128),         # 96 rows
     ([900, 300, 4100], 2, 6, 3, 128),          # 6 rows per KV head (warp-MMA kernel)
 ]
 

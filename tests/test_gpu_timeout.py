@@ -17,7 +17,7 @@ DEV = "cuda"
 TIMEOUT = 4   # SPIRE_DEVERR_TIMEOUT
 
 
-@pytest.mark.parametrize("kind", ["verify_tc", "verify_onecopy", "draft"])
+@pytest.mark.parametrize("kind", ["verify_tc", "verify_onecopy72", "verify_onecopy96", "draft"])
 def test_waits_run_out_then_the_next_call_is_correct(kind):
     import paper_2504_06419_gb300 as spire
     if kind == "draft":
@@ -34,7 +34,9 @@ def test_waits_run_out_then_the_next_call_is_correct(kind):
             return out
         ref, n_bad = parity.oracle_draft(inp)
     else:
-        hq, hkv, k = (32, 8, 4) if kind == "verify_tc" else (64, 8, 8)   # 20 / 72 rows per KV head
+        # 20 rows per KV head (four query copies), 72 and 96 (one copy)
+        hq, hkv, k = {"verify_tc": (32, 8, 4), "verify_onecopy72": (64, 8, 8),
+                      "verify_onecopy96": (64, 8, 11)}[kind]
         inp = wl.make_verify([3000, 700, 64 * 9 + 5, 2500], k, hq, hkv, 128, seed=92, device=DEV)
         desc = spire.verify_desc(inp.q, inp.k_cache, inp.block_table)
         ws = torch.empty(spire.spire_verify_workspace_bytes(desc, k), dtype=torch.uint8,
