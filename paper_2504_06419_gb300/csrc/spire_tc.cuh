@@ -4,7 +4,7 @@
 // Roles in a CTA (one CTA per SM, 7 warps):
 //   warp 0 (producer)   the TMA producer shared with the warp-MMA kernel:
 //                       K/V tiles into an NST-deep stage ring and each pair's
-//                       query rows into one of two Q buffers.
+//                       query rows into the Q buffer (one copy).
 //   warp 1 (QK issuer)  allocates tensor memory; one thread issues
 //                         S[sb]  = Q K^T   (M=128 rows, N=64 keys, K=D)
 //   warp 6 (PV issuer)  one thread issues
