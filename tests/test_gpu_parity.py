@@ -373,6 +373,33 @@ def test_split_plan_invariance(spire):
     assert rel <= 1e-5 and mx <= 1e-5, (rel, mx)
 
 
+@pytest.mark.parametrize("case", [(200000, 4, 4, 1), (100000, 8, 8, 1), (150000, 1, 32, 8)],
+                         ids=["four-copies", "one-copy", "eight-pairs"])
+def test_one_long_sequence_cut_across_every_sm(spire, case):
+    """A single sequence (one or a few pairs) cut into ~150 segments: every CTA
+    holds a piece of the same pair, and the completing CTA merges them all."""
+    L, k, Hq, Hkv = case
+    vi = wl.make_verify([L], k, Hq, Hkv, 128, seed=71, device=DEV, poison=True)
+    ws = torch.empty(spire.spire_verify_workspace_bytes(spire.verify_desc(vi.q, vi.k_cache,
+                                                                          vi.block_table), k),
+                     dtype=torch.uint8, device=DEV)
+    got = spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens, k,
+                                 workspace=ws)
+    assert spire.spire_get_device_error(ws) == 0
+    ref, n_bad = parity.oracle_verify(vi)
+    assert n_bad == 0
+    parity.assert_close(got.cpu().numpy(), ref, "one sequence, %s" % (case,))
+
+
+def test_draft_one_sequence_cut_into_one_tile_segments(spire):
+    """One pair of 8208 slots (129 tiles) over the SMs: a segment per tile."""
+    di = wl.make_draft([20000], 4, 1, 128, 16, 8192, seed=72, device=DEV, poison=True)
+    got = parity.gpu_draft(spire, di).cpu().numpy()
+    ref, n_bad = parity.oracle_draft(di)
+    assert n_bad == 0
+    parity.assert_close(got, ref, "draft, one sequence of 129 tiles")
+
+
 # ---------------------------------------------------------------- empty batches
 def test_every_call_accepts_an_empty_batch(spire):
     """B = 0 is a no-op for every call: empty results, no device error."""
