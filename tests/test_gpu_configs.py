@@ -1,13 +1,11 @@
 """Full-size parity on the benchmark workloads.
 
 Each call runs at full size in the same launch configuration the benchmark
-times.  The oracle then recomputes every sequence of the batch (the tiny,
-uniform 8K and ragged verify workloads, every draft workload), or, for the
-26 GB large-batch verify cache, a seeded sample of 24 sequences plus the
-shortest and the longest; every head and block row of them must match within
-max-abs 1e-2 and relative L2 1e-3, over the tensor and row by row.
+times.  The oracle then recomputes every sequence of the batch (the 26 GB
+large-batch verify cache 32 sequences at a time, each group's pages gathered
+on the device first); every head and block row must match within max-abs
+1e-2 and relative L2 1e-3, over the tensor and row by row.
 """
-import numpy as np
 import pytest
 import torch
 
@@ -24,14 +22,6 @@ def spire():
     return m
 
 
-def _sample(L, n, seed):
-    rng = np.random.default_rng(seed)
-    pick = set(rng.choice(len(L), size=min(n, len(L)), replace=False).tolist())
-    pick.add(int(np.argmin(L)))
-    pick.add(int(np.argmax(L)))
-    return sorted(pick)
-
-
 @pytest.mark.parametrize("name", ["tiny", "uniform8k", "ragged", "big"])
 def test_verify_full_config(spire, name):
     cfg = wl.CONFIGS[name]
@@ -44,21 +34,21 @@ def test_verify_full_config(spire, name):
     out = spire.verify_attention(vi.q, vi.k_cache, vi.v_cache, vi.block_table, vi.ctx_lens,
                                  cfg.k, workspace=ws)
     assert spire.spire_get_device_error(ws) == 0
-    if name == "big":
-        seqs = _sample(L, 24, cfg.seed)
-        sub = parity.compact_verify(vi, seqs)
-        got = out[torch.tensor(seqs, device=DEV)].cpu().numpy()
-    else:                      # the whole batch
-        seqs = list(range(len(L)))
-        sub = vi
-        got = out.cpu().numpy()
-    del out, ws
-    ref, n_bad = parity.oracle_verify(sub)
-    assert n_bad == 0
-    what = "verify %s (%s)" % (name, "all %d sequences" % len(L) if sub is vi else
-                               "sequences %s" % seqs)
-    parity.assert_close(got, ref, what)
-    del vi, sub
+    del ws
+    if name == "big":           # the whole batch, 32 sequences at a time
+        for g0 in range(0, len(L), 32):
+            seqs = list(range(g0, min(len(L), g0 + 32)))
+            sub = parity.compact_verify(vi, seqs)
+            got = out[g0:g0 + len(seqs)].cpu().numpy()
+            ref, n_bad = parity.oracle_verify(sub)
+            assert n_bad == 0
+            parity.assert_close(got, ref, "verify big (sequences %d..%d)" % (seqs[0], seqs[-1]))
+            del sub
+    else:                       # the whole batch at once
+        ref, n_bad = parity.oracle_verify(vi)
+        assert n_bad == 0
+        parity.assert_close(out.cpu().numpy(), ref, "verify %s (all %d sequences)" % (name, len(L)))
+    del vi, out
     torch.cuda.empty_cache()
 
 
