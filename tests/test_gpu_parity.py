@@ -42,6 +42,8 @@ VERIFY_CASES = [
     ([800, 333], 13, 10, 2, 128),              # 70 rows, G = 5
     ([500, 70, 3000], 11, 16, 2, 128),         # 96 rows
     ([900, 300, 4100], 2, 6, 3, 128),          # 6 rows per KV head (warp-MMA kernel)
+    ([300, 1000, 65], 1, 8, 2, 64),            # 8 rows at D = 64 (warp-MMA kernel)
+    ([1, 64, 2000], 0, 4, 4, 64),              # decoding, G = 1, D = 64 (warp-MMA kernel)
 ]
 
 
